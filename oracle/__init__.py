@@ -68,7 +68,7 @@ def lib():
         L = ctypes.CDLL(_build_lib())
         fp, i32, vp = ctypes.c_float, ctypes.c_int32, ctypes.c_void_p
         L.oracle_forward.argtypes = [ctypes.POINTER(OCfg), ctypes.POINTER(OWeights), vp, vp, i32,
-                                     vp, i32, vp, vp, i32, vp, vp]
+                                     vp, i32, vp, vp, i32, vp, vp, i32]
         L.oracle_forward.restype = ctypes.c_int
         L.oracle_matmul.argtypes = [vp, i32, i32, vp, i32, vp]
         L.oracle_matmul_cols.argtypes = [vp, i32, i32, vp, vp, i32, vp]

@@ -8,8 +8,10 @@
  * (Eq. 6), the target verification pass (Section 2.2) and autoregressive
  * greedy decoding (Eq. 2).
  *
- * Weights are bf16 bit patterns, widened exactly to fp32 when read.  All
- * arithmetic is fp32, compiled with -ffp-contract=off (no fused multiply-add),
+ * Weights are bf16 bit patterns, widened exactly to fp32 when read.  The
+ * paper runs its models in bf16 (Table 3), so the KV cache stores bf16
+ * values: with kv_bf16 set, each key and value is rounded to bf16
+ * (round-to-nearest-even) when it enters the cache.  All arithmetic is fp32, compiled with -ffp-contract=off (no fused multiply-add),
  * so results are identical on every IEEE host.  Every dot product is summed
  * in the same order whatever the number of rows computed together, so a row
  * computed inside a batch is bitwise equal to the same row computed alone.
@@ -48,6 +50,16 @@ typedef struct {
 static inline float bf16_to_f32(uint16_t b) {
   union { uint32_t u; float f; } v;
   v.u = (uint32_t)b << 16;
+  return v.f;
+}
+
+/* fp32 -> nearest bf16 (ties to even), returned widened to fp32 */
+static inline float round_bf16(float f) {
+  union { float f; uint32_t u; } v;
+  v.f = f;
+  if ((v.u & 0x7F800000u) == 0x7F800000u) return f;
+  v.u += 0x7FFFu + ((v.u >> 16) & 1u);
+  v.u &= 0xFFFF0000u;
   return v.f;
 }
 
@@ -155,10 +167,11 @@ static inline float silu(float z) { return z / (1.0f + expf(-z)); }
  *           every position <= max(pos) must be cached or among the new rows.
  *   out_rows[n_out]: rows whose logits are written to logits[n_out][vocab]
  *   hidden (optional): final-norm input h, [m][d].
+ *   kv_bf16: store keys and values rounded to bf16 (else as fp32).
  */
 int oracle_forward(const ocfg* c, const oweights* w, float* kc, float* vc, int32_t max_pos,
                    const int32_t* tokens, int32_t m, const int32_t* pos,
-                   const int32_t* out_rows, int32_t n_out, float* logits, float* hidden) {
+                   const int32_t* out_rows, int32_t n_out, float* logits, float* hidden, int32_t kv_bf16) {
   const int32_t d = c->d, hq = c->hq, hkv = c->hkv, hd = c->hd, ffn = c->ffn;
   const int32_t qd = hq * hd, kvd = hkv * hd, group = hq / hkv;
   for (int32_t i = 0; i < m; ++i) {
@@ -189,8 +202,11 @@ int oracle_forward(const ocfg* c, const oweights* w, float* kc, float* vc, int32
     for (int32_t i = 0; i < m; ++i) {
       for (int32_t hh = 0; hh < hq; ++hh) oracle_rope(q + (int64_t)i * qd + hh * hd, hd, pos[i], c->theta);
       for (int32_t hh = 0; hh < hkv; ++hh) oracle_rope(k + (int64_t)i * kvd + hh * hd, hd, pos[i], c->theta);
-      memcpy(kl + (int64_t)pos[i] * kvd, k + (int64_t)i * kvd, sizeof(float) * kvd);
-      memcpy(vl + (int64_t)pos[i] * kvd, v + (int64_t)i * kvd, sizeof(float) * kvd);
+      for (int32_t e = 0; e < kvd; ++e) {
+        const float ke = k[(int64_t)i * kvd + e], ve = v[(int64_t)i * kvd + e];
+        kl[(int64_t)pos[i] * kvd + e] = kv_bf16 ? round_bf16(ke) : ke;
+        vl[(int64_t)pos[i] * kvd + e] = kv_bf16 ? round_bf16(ve) : ve;
+      }
     }
 #pragma omp parallel
     {

@@ -37,11 +37,14 @@ from .philox import (STREAM_ACCEPT, STREAM_BONUS, STREAM_DRAFT, gumbel, raw_word
 
 
 class OracleModel:
-    """One decoder (target or draft) with a per-sequence fp32 KV cache."""
+    """One decoder (target or draft) with a per-sequence KV cache.  The cache
+    holds bf16 values (the paper's model precision, Table 3) unless
+    ``kv_bf16=False``, which keeps fp32 keys and values."""
 
-    def __init__(self, shape, weights: dict, batch: int, max_pos: int):
+    def __init__(self, shape, weights: dict, batch: int, max_pos: int, kv_bf16: bool = True):
         self.shape = shape
         self.max_pos = max_pos
+        self.kv_bf16 = bool(kv_bf16)
         self.cfg = OCfg(shape.n_layers, shape.d_model, shape.n_q_heads, shape.n_kv_heads,
                         shape.head_dim, shape.ffn, shape.vocab, shape.rope_theta, shape.rms_eps)
         self._keep = []
@@ -74,7 +77,8 @@ class OracleModel:
         rc = lib().oracle_forward(ctypes.byref(self.cfg), ctypes.byref(self.w),
                                   self.kc[b].ctypes.data, self.vc[b].ctypes.data, self.max_pos,
                                   tok.ctypes.data, m, pos.ctypes.data, rows.ctypes.data, len(rows),
-                                  logits.ctypes.data, hidden.ctypes.data if want_hidden else None)
+                                  logits.ctypes.data, hidden.ctypes.data if want_hidden else None,
+                                  int(self.kv_bf16))
         if rc != 0:
             raise ValueError(f"oracle_forward rejected its arguments (code {rc})")
         logits = logits[:len(rows)]
@@ -197,11 +201,13 @@ class OracleDecoder:
         draft pending = [x_P]."""
         wl = self.wl
         self.n, self.pending, self.generated, self.done = [], [], [], []
+        self.prefill_logits = []
         first = []
         for b, pr in enumerate(prompts):
             P = len(pr)
             pos = np.arange(P, dtype=np.int32)
             lg = self.T.forward(b, pr, pos, [P - 1])[0]
+            self.prefill_logits.append(lg)
             self.D.forward(b, pr, pos, [])
             if wl.sample:
                 zT = (lg / np.float32(wl.temperature)).astype(np.float32)
@@ -213,8 +219,12 @@ class OracleDecoder:
             self.pending.append([x])
             self.generated.append([x])
             self.done.append(wl.n_new <= 1)
-        self.prefill_logits_last = None
         return first
+
+    def force_first(self, b: int, tok: int) -> None:
+        """Teacher forcing: replace sequence b's first generated token."""
+        self.pending[b] = [int(tok)]
+        self.generated[b] = [int(tok)]
 
     # -- one step -----------------------------------------------------------
     def draft(self, step: int, seed: int = 0) -> Tuple[np.ndarray, np.ndarray]:
@@ -308,10 +318,10 @@ class OracleDecoder:
         return self.generated, trace
 
 
-def ar_greedy(shape, weights: dict, prompt: Sequence[int], n_new: int) -> List[int]:
+def ar_greedy(shape, weights: dict, prompt: Sequence[int], n_new: int, kv_bf16: bool = True) -> List[int]:
     """Eq. 2: x_t = argmax P(x | x_0..x_{t-1}), one target forward per token."""
     P = len(prompt)
-    m = OracleModel(shape, weights, 1, P + n_new + 1)
+    m = OracleModel(shape, weights, 1, P + n_new + 1, kv_bf16)
     lg = m.forward(0, prompt, np.arange(P, dtype=np.int32), [P - 1])[0]
     out = [argmax_lowest(lg)]
     while len(out) < n_new:

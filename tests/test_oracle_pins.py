@@ -156,7 +156,7 @@ def test_forward_matches_library_model_prefill_and_incremental(tiny):
     wl, tw, _ = tiny
     toks = wl.prompts()[0].tolist() + [5, 77, 2047, 1000]
     ref = torch_llama_logits(wl.target, tw, toks)
-    m = P.OracleModel(wl.target, tw, 1, 64)
+    m = P.OracleModel(wl.target, tw, 1, 64, kv_bf16=False)
     P0 = 32
     pre = m.forward(0, toks[:P0], list(range(P0)), list(range(P0)))
     assert np.abs(pre - ref[:P0]).max() < 2e-4
@@ -167,6 +167,26 @@ def test_forward_matches_library_model_prefill_and_incremental(tiny):
     inc = np.concatenate([r1, r2, r3])
     assert np.abs(inc - ref[P0:]).max() < 2e-4
     assert np.abs(ref).max() > 0.5                # not a degenerate all-zero model
+
+
+def test_bf16_cache_stores_rounded_fp32_values(tiny):
+    """With the bf16 cache, every stored key/value is the round-to-nearest-even
+    bf16 value of the fp32 one, and logits stay within bf16-storage error."""
+    wl, tw, _ = tiny
+    toks = wl.prompts()[0].tolist()
+    a = P.OracleModel(wl.target, tw, 1, 40, kv_bf16=False)
+    b = P.OracleModel(wl.target, tw, 1, 40, kv_bf16=True)
+    la = a.forward(0, toks[:1], [0], [0])
+    lb = b.forward(0, toks[:1], [0], [0])
+    # one row: attention reads only its own key/value, so layer 0's cache entry is comparable exactly
+    k32 = a.kc[0][0, 0].astype(np.float32)
+    u = k32.view(np.uint32).astype(np.uint64)
+    rne = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16 << 16).astype(np.uint32).view(np.float32)
+    assert np.array_equal(b.kc[0][0, 0], rne)
+    assert np.abs(la - lb).max() < 0.05 * np.abs(la).max()
+    la = a.forward(0, toks[1:], range(1, len(toks)), range(len(toks) - 1))
+    lb = b.forward(0, toks[1:], range(1, len(toks)), range(len(toks) - 1))
+    assert 0 < np.abs(la - lb).max() < 0.05 * np.abs(la).max()
 
 
 def test_forward_rejects_bad_arguments(tiny):
