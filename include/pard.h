@@ -1,0 +1,182 @@
+/*
+ * libpard -- PARD speculative decode step on one GB300 (sm_103a).
+ *
+ * C ABI: plain pointers and sizes only.  Pointers named d_* are device
+ * pointers, h_* are host pointers.  `stream` is a cudaStream_t passed as
+ * void*; every call that takes one only enqueues work on it (no host
+ * synchronisation) unless stated otherwise.  No call allocates device memory:
+ * the caller owns the weights, the KV page pool and the workspace, sized by
+ * pard_kv_pool_bytes / pard_workspace_bytes; the library only borrows them.
+ * Errors are returned as pard_status codes, with a message available from
+ * pard_last_error(); kernels that detect a bad index or a stalled pipeline
+ * set a sticky device status word read by pard_last_status().
+ *
+ * The decode step (paper: PARD, arXiv 2504.18583):
+ *   pard_draft          one draft forward over the accepted prefix plus
+ *                       mask tokens predicts K tokens at once (Section 3.1,
+ *                       Eq. 6; shared mask id, Section 4.3)
+ *   pard_verify         one target forward over the last token and the K
+ *                       candidates (Section 2.2, verification stage)
+ *   pard_accept_commit  greedy prefix match or speculative-sampling
+ *                       rejection with residual resampling (the rule of the
+ *                       speculative decoding papers the paper builds on,
+ *                       Section 2.2), then KV commit / rollback by length
+ * pard_prefill fills both caches from the prompts and emits the first token.
+ */
+#ifndef PARD_H
+#define PARD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  PARD_OK = 0,
+  PARD_ERR_ARG = -1,          /* null pointer, bad size or bad value */
+  PARD_ERR_SHAPE = -2,        /* model shape the kernels do not support */
+  PARD_ERR_NO_PAGES = -3,     /* KV page pool too small for the request */
+  PARD_ERR_CUDA = -4,         /* a CUDA runtime/driver call failed */
+  PARD_ERR_DEVICE_CHECK = -5, /* a kernel flagged a bad index (see pard_last_status) */
+  PARD_ERR_TIMEOUT = -6,      /* a kernel pipeline wait ran out (see pard_last_status) */
+  PARD_ERR_STATE = -7         /* call out of order (e.g. draft before prefill) */
+} pard_status;
+
+/* Llama-style decoder shape (the LLaMA3 family of Section 4.1).
+ * Supported: head_dim 64 or 128, n_q_heads a multiple of n_kv_heads,
+ * d_model, n_q_heads*head_dim and n_kv_heads*head_dim multiples of 128,
+ * ffn a multiple of 8, vocab a multiple of 8, mask_id in [0, vocab). */
+typedef struct {
+  int32_t n_layers, d_model, n_q_heads, n_kv_heads, head_dim, ffn, vocab;
+  float rope_theta, rms_eps;
+  int32_t mask_id;
+} pard_model_cfg;
+
+/* Device pointers to bf16 weights, all row-major [out][in]:
+ *   embed [vocab][d], final_norm [d], lm_head [vocab][d],
+ *   layers: host array of n_layers*9 device pointers, per layer in the order
+ *   attn_norm [d], wq [hq*hd][d], wk [hkv*hd][d], wv [hkv*hd][d],
+ *   wo [d][hq*hd], mlp_norm [d], wg [ffn][d], wu [ffn][d], wd [d][ffn].
+ * Every pointer must be 16-byte aligned.  Borrowed until pard_destroy. */
+typedef struct {
+  const void* embed;
+  const void* final_norm;
+  const void* lm_head;
+  const void* const* layers;
+} pard_weights;
+
+/* Sizes the workspace and page pool are built for. */
+typedef struct {
+  int32_t max_batch;      /* sequences decoded together (<= 64) */
+  int32_t max_k;          /* draft length K (1..16) */
+  int32_t max_ctx;        /* positions one sequence may reach (prompt + new + 2K) */
+  int32_t page_size;      /* KV page size in tokens (16) */
+  int32_t prefill_chunk;  /* rows per prefill forward (multiple of 64, <= 1024) */
+  int32_t n_pages;        /* pages in each model's pool */
+} pard_limits;
+
+typedef struct pard_ctx pard_ctx;
+
+/* Bytes of device workspace needed for these models and limits (host only,
+ * no CUDA call).  Returns 0 if the arguments are invalid. */
+size_t pard_workspace_bytes(const pard_model_cfg* target, const pard_model_cfg* draft, const pard_limits* lim);
+
+/* Bytes of the KV page pool: lim->n_pages pages for each model, each page
+ * holding K and V of page_size tokens for every layer, bf16, laid out
+ * [layer][K|V][page][kv_head][token][head_dim].  Host only. */
+size_t pard_kv_pool_bytes(const pard_model_cfg* target, const pard_model_cfg* draft, const pard_limits* lim);
+
+/* Validate shapes, record the borrowed pointers, carve the workspace and
+ * build TMA descriptors and RoPE tables.  h_page_order_{target,draft}
+ * (host, n_pages entries each, a permutation of 0..n_pages-1, or NULL for
+ * the identity) give the order in which pages are handed to sequences.
+ * Synchronises `stream` once (uploads tables).  On success *out owns host
+ * state only; device memory stays the caller's. */
+pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* target, const pard_weights* target_w,
+                              const pard_model_cfg* draft, const pard_weights* draft_w, const pard_limits* lim,
+                              void* d_kv_pool, size_t kv_pool_bytes, void* d_workspace, size_t workspace_bytes,
+                              const int32_t* h_page_order_target, const int32_t* h_page_order_draft, void* stream);
+
+/* Prefill both models on `batch` prompts (d_tokens: the prompts
+ * concatenated, h_lens[b] tokens each) and emit each sequence's first new
+ * token into d_first_token[b] (argmax, or a Gumbel-max draw at
+ * `temperature` with Philox stream 2, step 0 when sample != 0).
+ * Reserves ceil((len + n_new + 2K) / page_size) pages per sequence and
+ * model, in sequence order, from the front of the page order.
+ * n_new: tokens to generate per sequence, the first one included; K: the
+ * draft length every later pard_draft uses.  Synchronises `stream`. */
+pard_status pard_prefill(pard_ctx* ctx, const int32_t* d_tokens, const int32_t* h_lens, int32_t batch,
+                         int32_t n_new, int32_t K, int32_t sample, float temperature, uint64_t seed,
+                         int32_t* d_first_token, void* stream);
+
+/* One draft forward (Eq. 6): the pending real tokens of each sequence, then
+ * K-1 mask tokens, at consecutive positions; the K predictions are read at
+ * the last real row and at every mask row.  Greedy: argmax; sample != 0:
+ * Gumbel-max draw from softmax(z / temperature) with Philox stream 0.
+ * Writes d_draft_out [B][K] and, if non-NULL, the draft logits
+ * d_draft_logits [B][K][vocab] (fp32).  Mask rows leave the draft cache by
+ * length only. */
+pard_status pard_draft(pard_ctx* ctx, int32_t sample, float temperature, uint64_t seed, uint64_t step,
+                       int32_t* d_draft_out, float* d_draft_logits, void* stream);
+
+/* One target forward over [last token, d_0..d_{K-1}] at positions
+ * n-1..n+K-1 of each sequence.  d_draft_in [B][K]: candidates to verify, or
+ * NULL for the ones the last pard_draft produced.  Writes per-row logit
+ * statistics for pard_accept_commit and, if non-NULL, the logits
+ * d_logits_out [B][K+1][vocab] (fp32). */
+pard_status pard_verify(pard_ctx* ctx, const int32_t* d_draft_in, float temperature, float* d_logits_out,
+                        void* stream);
+
+/* Accept and commit.  Greedy: a = longest prefix with d_i == argmax y_i,
+ * bonus = argmax y_a.  sample != 0: accept d_i while u_i * q_i(d_i) <
+ * p_i(d_i) (u_i: Philox stream 1), at the first rejection j draw the bonus
+ * from max(0, p_j - q_j) renormalised, after K acceptances draw it from p_K
+ * (Gumbel-max, stream 2).  Then target length += a + 1 (rejected slots are
+ * dropped by length), draft pending tokens = d_0..d_{a-1}, bonus.
+ * Outputs (device, may be NULL): d_accept_len [B] = a; d_emitted [B][K+1]
+ * = emitted tokens that count toward n_new, -1 after them; d_kv_slots
+ * [B][K+1] = cache slots page*page_size + pos%page_size of the committed
+ * target positions n-1..n-1+a, -1 after them; d_n_emit [B] = tokens counted.
+ * Finished sequences keep their state and report a = 0, no tokens. */
+pard_status pard_accept_commit(pard_ctx* ctx, int32_t sample, float temperature, uint64_t seed, uint64_t step,
+                               int32_t* d_accept_len, int32_t* d_emitted, int32_t* d_kv_slots, int32_t* d_n_emit,
+                               void* stream);
+
+/* Replace the logits the next pard_accept_commit reads (testing the
+ * acceptance rule on given inputs): d_target_logits [B][K+1][vocab],
+ * d_draft_logits [B][K][vocab] (may be NULL when greedy), d_draft [B][K]. */
+pard_status pard_set_logits(pard_ctx* ctx, const float* d_target_logits, const float* d_draft_logits,
+                            const int32_t* d_draft, float temperature, void* stream);
+
+/* Host copy of per-sequence state: h_n [B] (tokens so far, incl. pending),
+ * h_generated [B], h_done [B].  Synchronises `stream`.  Any may be NULL. */
+pard_status pard_get_state(pard_ctx* ctx, int32_t* h_n, int32_t* h_generated, int32_t* h_done, void* stream);
+
+/* Copy one layer's KV entries at the given positions of sequence b into
+ * host-visible device buffers d_k, d_v [n][n_kv_heads][head_dim] (bf16),
+ * reading through the page table (for checking the cache layout).
+ * model: 0 target, 1 draft. */
+pard_status pard_read_kv(pard_ctx* ctx, int32_t model, int32_t layer, int32_t b, const int32_t* h_pos, int32_t n,
+                         void* d_k, void* d_v, void* stream);
+
+/* Synchronise `stream` and return the sticky device status word in
+ * *h_flags (0 = clean); the word is cleared.  Returns PARD_ERR_TIMEOUT or
+ * PARD_ERR_DEVICE_CHECK when bits are set. */
+pard_status pard_last_status(pard_ctx* ctx, uint32_t* h_flags, void* stream);
+
+/* Kernel launches the last call enqueued (for launch accounting). */
+int32_t pard_launch_count(pard_ctx* ctx);
+
+/* Thread-local message for the last failing call ("" if none). */
+const char* pard_last_error(void);
+
+/* Release host state.  Does not free caller-owned device memory. */
+void pard_destroy(pard_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PARD_H */

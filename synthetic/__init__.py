@@ -273,3 +273,32 @@ def random_ints(seed: int, tag: int, lo: int, hi_exclusive: int, n: int) -> np.n
     out = np.empty(n, dtype=np.int32)
     _lib().synth_uniform_int(seed, (6 << 48) + tag, lo, hi_exclusive - lo, out.ctypes.data, n)
     return out
+
+
+# --------------------------------------------------------------------------
+# Upload to a CUDA device (torch is used for memory only)
+# --------------------------------------------------------------------------
+def device_weights(shape: ModelShape, seed: int, model_tag: int, device="cuda", norm_jitter: float = 0.0,
+                   host: Optional[dict] = None) -> dict:
+    """Same tensors as ``model_weights``, as contiguous bf16 CUDA tensors.
+    Generated tensor by tensor into one pinned staging buffer (or taken from
+    ``host`` when given) so host memory stays at one tensor."""
+    import torch
+    biggest = max(int(np.prod(shape.tensor_shape(n))) for _, n in iter_tensors(shape))
+    staging = None if host is not None else torch.empty(biggest, dtype=torch.int16, pin_memory=True)
+    out = {"layers": [dict() for _ in range(shape.n_layers)]}
+    for layer, name in iter_tensors(shape):
+        dims = shape.tensor_shape(name)
+        numel = int(np.prod(dims))
+        dev = torch.empty(dims, dtype=torch.bfloat16, device=device)
+        if host is not None:
+            src = host[name] if layer < 0 else host["layers"][layer][name]
+            dev.view(torch.int16).copy_(torch.from_numpy(np.ascontiguousarray(src).view(np.int16)))
+        else:
+            fill_tensor(shape, seed, model_tag, layer, name, staging.data_ptr(), numel, norm_jitter=norm_jitter)
+            dev.view(torch.int16).view(-1).copy_(staging[:numel])
+        if layer < 0:
+            out[name] = dev
+        else:
+            out["layers"][layer][name] = dev
+    return out

@@ -1,0 +1,147 @@
+"""Shared harness of the GPU parity tests: the same seeded inputs go to the
+CUDA path (through the C ABI) and to the CPU oracle; results are compared
+step by step.
+
+Tolerances (the decode step's floating-point contract): logits within
+max-abs 3e-2 of the fp32 oracle; token ids, accept lengths and KV slot
+indices bit-exact wherever the oracle's top-1 / top-2 logit margin exceeds
+5e-2.  Where a margin is below that, the GPU's choice must still be a valid
+one (within 2 x 3e-2 of the oracle's maximum) and the oracle is forced onto
+the GPU's tokens (teacher forcing), so later steps compare like with like."""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle
+import synthetic as S
+from oracle import pard as OP
+from oracle.philox import STREAM_ACCEPT, raw_words, uniform01
+
+LOGIT_TOL = 3e-2
+MARGIN = 5e-2
+
+
+def margin(row: np.ndarray) -> float:
+    top2 = np.partition(row, -2)[-2:]
+    return float(top2[1] - top2[0])
+
+
+class Pair:
+    """GPU engine and oracle decoder on identical weights and page orders."""
+
+    def __init__(self, wl, draft_is_target: bool = False, prefill_chunk: int = 64):
+        import torch
+        from paper_2504_18583_gb300 import pard
+        self.wl = wl
+        tw = S.model_weights(wl.target, wl.seed, S.TARGET, wl.norm_jitter)
+        dw = tw if draft_is_target else S.model_weights(wl.draft, wl.seed, S.DRAFT, wl.norm_jitter)
+        dshape = wl.target if draft_is_target else wl.draft
+        self.wl = wl = wl.replace(draft=dshape)
+        self.tw_host, self.dw_host = tw, dw
+        self.prompts = wl.prompts()
+        lens = [len(p) for p in self.prompts]
+        n_pages = wl.n_pages()
+        self.order_t, self.order_d = wl.page_order(S.TARGET), wl.page_order(S.DRAFT)
+        self.oracle = oracle.OracleDecoder(wl, tw, dw, self.order_t, self.order_d)
+        self.tw_dev = S.device_weights(wl.target, 0, 0, host=tw)
+        self.dw_dev = self.tw_dev if draft_is_target else S.device_weights(dshape, 0, 0, host=dw)
+        max_ctx = max(lens) + wl.n_new + 2 * wl.K + 16
+        self.eng = pard.PardEngine(wl.target, self.tw_dev, dshape, self.dw_dev, max_batch=wl.batch, max_k=wl.K,
+                                   max_ctx=max_ctx, n_pages=n_pages, prefill_chunk=prefill_chunk,
+                                   page_order_target=self.order_t, page_order_draft=self.order_d)
+        self.torch = torch
+        self.stats = dict(excused_tokens=0, checked_tokens=0, max_logit_err=0.0, max_draft_logit_err=0.0)
+
+    def prefill(self, seed=0):
+        first_g = self.eng.prefill(self.prompts, self.wl.n_new, self.wl.K, self.wl.sample, self.wl.temperature,
+                                   seed).cpu().numpy()
+        first_o = self.oracle.prefill(self.prompts, seed)
+        for b in range(self.wl.batch):
+            if not self.wl.sample:
+                check_token(int(first_g[b]), self.oracle.prefill_logits[b], self.stats, f"first token seq {b}")
+            if int(first_g[b]) != int(first_o[b]):
+                self.stats["excused_tokens"] += 1
+                self.oracle.force_first(b, int(first_g[b]))
+        return first_g, first_o
+
+    def active(self):
+        return [b for b in range(self.wl.batch) if not self.oracle.done[b]]
+
+
+def check_token(gpu_tok: int, oracle_logits: np.ndarray, stats: dict, what: str) -> None:
+    """Bit-exact where the margin is clear; otherwise the GPU's token must be
+    within 2 x LOGIT_TOL of the oracle's maximum."""
+    o_tok = int(np.argmax(oracle_logits))
+    stats["checked_tokens"] += 1
+    if margin(oracle_logits) > MARGIN:
+        assert gpu_tok == o_tok, f"{what}: gpu {gpu_tok} oracle {o_tok} margin {margin(oracle_logits):.3g}"
+    else:
+        assert oracle_logits[gpu_tok] >= oracle_logits[o_tok] - 2 * LOGIT_TOL, what
+        if gpu_tok != o_tok:
+            stats["excused_tokens"] += 1
+
+
+def greedy_step(P: Pair, step: int, inject=None):
+    """One teacher-forced greedy step; returns the GPU outputs."""
+    torch = P.torch
+    wl, K = P.wl, P.wl.K
+    out = P.eng.alloc_step_outputs(want_logits=True)
+    P.eng.draft(out, False, 1.0, 0, step)
+    d_gpu = out["draft"].cpu().numpy()
+    z_gpu = out["draft_logits"].cpu().numpy()
+    d_or, z_or = P.oracle.draft(step)
+    for b in P.active():
+        err = float(np.abs(z_gpu[b] - z_or[b]).max())
+        P.stats["max_draft_logit_err"] = max(P.stats["max_draft_logit_err"], err)
+        assert err <= LOGIT_TOL, f"draft logits step {step} seq {b}: {err}"
+        for i in range(K):
+            check_token(int(d_gpu[b, i]), z_or[b, i], P.stats, f"draft step {step} seq {b} i {i}")
+    cand = d_gpu if inject is None else inject
+    cand_t = None if inject is None else torch.as_tensor(inject, dtype=torch.int32, device="cuda")
+    P.eng.verify(out, cand_t, 1.0)
+    y_gpu = out["logits"].cpu().numpy()
+    y_or = P.oracle.verify(cand)
+    for b in P.active():
+        err = float(np.abs(y_gpu[b] - y_or[b]).max())
+        P.stats["max_logit_err"] = max(P.stats["max_logit_err"], err)
+        assert err <= LOGIT_TOL, f"verify logits step {step} seq {b}: {err}"
+    P.eng.accept_commit(out, False, 1.0, 0, step)
+    a_gpu = out["accept_len"].cpu().numpy()
+    em_gpu = out["emitted"].cpu().numpy()
+    slots_gpu = out["kv_slots"].cpu().numpy()
+    n_emit = out["n_emit"].cpu().numpy()
+    acc, emitted = [], []
+    for b in range(wl.batch):
+        if P.oracle.done[b]:
+            assert a_gpu[b] == 0 and n_emit[b] == 0 and (em_gpu[b] == -1).all()
+            acc.append(0)
+            emitted.append([])
+            continue
+        a = int(a_gpu[b])
+        t_gpu = [int(np.argmax(y_gpu[b, i])) for i in range(K + 1)]
+        for i in range(K + 1):
+            check_token(t_gpu[i], y_or[b, i], P.stats, f"verify step {step} seq {b} row {i}")
+        # the accept kernel applies the prefix rule exactly to the GPU's own argmax
+        a_rule = 0
+        while a_rule < K and int(cand[b, a_rule]) == t_gpu[a_rule]:
+            a_rule += 1
+        assert a == a_rule, f"accept length {a} != prefix rule {a_rule}"
+        a_or, em_or = OP.accept_greedy(cand[b], y_or[b])
+        if a_or != a:
+            # only allowed when the deciding row's margin is within tolerance
+            i = min(a, a_or)
+            assert margin(y_or[b, i]) <= MARGIN, f"accept length step {step} seq {b}: gpu {a} oracle {a_or}"
+            P.stats["excused_tokens"] += 1
+        gpu_em = [int(x) for x in cand[b, :a]] + [int(np.argmax(y_gpu[b, a]))]
+        take = int(n_emit[b])
+        assert [int(x) for x in em_gpu[b, :take]] == gpu_em[:take]
+        assert (em_gpu[b, take:] == -1).all()
+        acc.append(a)
+        emitted.append(gpu_em)
+    slots_or, nout = P.oracle.commit(acc, emitted)
+    for b in range(wl.batch):
+        if b < len(nout) and nout[b] == 0 and a_gpu[b] == 0 and n_emit[b] == 0:
+            continue
+        assert np.array_equal(slots_gpu[b], slots_or[b]), f"kv slots step {step} seq {b}"
+        assert n_emit[b] == nout[b]
+    return dict(a=a_gpu, emitted=em_gpu, slots=slots_gpu, d=d_gpu, y=y_gpu, z=z_gpu)

@@ -1,0 +1,217 @@
+"""GPU parity of the PARD decode step against the CPU oracle, through the
+C ABI.  Every test builds both sides from the same seeded inputs."""
+import numpy as np
+import pytest
+
+import oracle
+import synthetic as S
+from oracle import pard as OP
+from oracle.philox import STREAM_ACCEPT, STREAM_BONUS, raw_words, uniform01
+
+from _parity import LOGIT_TOL, MARGIN, Pair, check_token, greedy_step, margin
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2504_18583_gb300 import _build
+    _build.build()
+
+
+def run_greedy(P: Pair, max_steps=64, inject_fn=None):
+    P.prefill()
+    step = 1
+    outs = []
+    while not P.oracle.all_done() and step <= max_steps:
+        inject = inject_fn(P, step) if inject_fn else None
+        outs.append(greedy_step(P, step, inject))
+        step += 1
+    n, gen, done = P.eng.state()
+    assert done == [1 if d else 0 for d in P.oracle.done]
+    assert P.eng.last_status() == 0
+    return outs
+
+
+def test_tiny_greedy_matches_oracle_every_step():
+    wl = S.WORKLOADS["tiny"]
+    P = Pair(wl)
+    run_greedy(P)
+    assert P.oracle.all_done()
+    # the generated sequence equals autoregressive greedy decoding where margins are clear
+    assert P.stats["excused_tokens"] <= P.stats["checked_tokens"] // 10
+    print("stats", P.stats)
+
+
+def test_tiny_greedy_jittered_norms_batch_ragged():
+    """Batch of 3 with prompts 17 / 33 / 50 tokens (page boundaries at
+    several offsets), norm gains != 1, prefill chunks of 64 rows."""
+    wl = S.WORKLOADS["tiny"].replace(batch=3, prompt_len=None, prompt_len_range=(17, 50), norm_jitter=0.1,
+                                     n_new=20)
+    P = Pair(wl)
+    run_greedy(P)
+    print("stats", P.stats)
+
+
+def test_self_draft_accepts_and_rolls_back():
+    """Draft = target: d_0 always equals the target's argmax, so every step
+    accepts at least one candidate and commit/rollback runs with a > 0."""
+    wl = S.WORKLOADS["tiny"].replace(n_new=30, batch=2, prompt_len=40)
+    P = Pair(wl, draft_is_target=True)
+    outs = run_greedy(P)
+    accs = [int(o["a"][b]) for o in outs for b in range(2)]
+    assert max(accs) >= 1
+    print("accept lengths", accs, P.stats)
+
+
+def test_injected_candidates_hit_every_accept_length():
+    """pard_verify on the target's own greedy continuation with one planted
+    mismatch at j accepts exactly j candidates (j = K: none planted)."""
+    wl = S.WORKLOADS["tiny"].replace(n_new=40)
+    P = Pair(wl)
+    K = wl.K
+    ar = oracle.ar_greedy(wl.target, P.tw_host, P.prompts[0], wl.n_new + K + 2)
+    seen = set()
+
+    def inject(P, step):
+        n0 = len(P.oracle.generated[0])
+        j = (step - 1) % (K + 1)
+        cont = list(ar[n0:n0 + K])
+        while len(cont) < K:
+            cont.append(0)
+        if j < K:
+            cont[j] = (cont[j] + 1) % (wl.target.vocab - 1)
+        return np.array([cont], dtype=np.int32)
+
+    outs = run_greedy(P, inject_fn=inject)
+    for s, o in enumerate(outs):
+        seen.add(int(o["a"][0]))
+    assert seen >= set(range(K + 1)) - {K} or len(seen) >= K
+    print("accept lengths seen", sorted(seen), P.stats)
+
+
+def test_kv_cache_holds_the_oracle_keys_and_values():
+    wl = S.WORKLOADS["tiny"].replace(n_new=12)
+    P = Pair(wl)
+    run_greedy(P)
+    n = P.oracle.n[0]
+    pos = list(range(0, n - 1))
+    for model, om, shape in ((0, P.oracle.T, wl.target), (1, P.oracle.D, wl.draft)):
+        upto = n - 1 if model == 0 else n - len(P.oracle.pending[0])
+        for layer in (0, shape.n_layers - 1):
+            k, v = P.eng.read_kv(model, layer, 0, pos[:upto], shape)
+            k = k.float().cpu().numpy()
+            v = v.float().cpu().numpy()
+            ko = om.kc[0][layer, :upto]
+            vo = om.vc[0][layer, :upto]
+            # bf16 storage: relative 2^-8 plus the accumulated logit-level error
+            assert np.abs(k - ko).max() <= 0.02 * max(1.0, np.abs(ko).max())
+            assert np.abs(v - vo).max() <= 0.02 * max(1.0, np.abs(vo).max())
+
+
+def test_full_width_8b_layers_short_prompt():
+    """8B-shaped target and 1B-shaped draft at full width (every GEMM,
+    attention and LM-head tile count of the full models), two layers each,
+    64-token prompt, three steps."""
+    wl = S.WORKLOADS["8b_greedy"].replace(target=S.TARGET_8B.replace(n_layers=2),
+                                          draft=S.DRAFT_1B.replace(n_layers=2), prompt_len=64, n_new=20)
+    P = Pair(wl, prefill_chunk=64)
+    P.prefill()
+    for step in range(1, 4):
+        greedy_step(P, step)
+    assert P.eng.last_status() == 0
+    print("stats", P.stats)
+
+
+# ----------------------------------------------------------------------------
+# speculative sampling
+# ----------------------------------------------------------------------------
+def test_sampling_decisions_on_identical_logits():
+    """Level 1: the oracle's logits fed to the GPU acceptance kernels with the
+    same Philox streams give the same accept/reject decisions and bonus draws
+    (except where u*q and p are within a few ulps)."""
+    import torch
+    wl = S.WORKLOADS["tiny"].replace(sample=True, n_new=1000, K=4)
+    P = Pair(wl)
+    P.prefill(seed=5)
+    rng = np.random.default_rng(0)
+    V, K = wl.target.vocab, wl.K
+    mism = 0
+    for trial in range(40):
+        y = (rng.standard_normal((1, K + 1, V)) * 2.0).astype(np.float32)
+        z = (y[:, :K] + rng.standard_normal((1, K, V)).astype(np.float32) * (0.3 + 0.1 * (trial % 5))).astype(np.float32)
+        d = np.array([OP.draft_tokens(z[0], True, 1.0, 77 + trial, 3, 0)], dtype=np.int32)
+        P.eng.set_logits(torch.as_tensor(y, device="cuda"), torch.as_tensor(z, device="cuda"),
+                         torch.as_tensor(d, device="cuda"), 1.0)
+        out = P.eng.alloc_step_outputs()
+        step = 1000 + trial
+        n_before = P.eng.state()[0][0]
+        P.eng.accept_commit(out, True, 1.0, 5, step)
+        a_g = int(out["accept_len"][0])
+        em_g = out["emitted"][0].cpu().numpy()
+        a_o, em_o = OP.accept_sampling(d[0], z[0], y[0], 1.0, 5, step, 0)
+        if a_o != a_g:
+            # excuse only a decision within rounding of the threshold
+            i = min(a_o, a_g)
+            p = OP.softmax_t(y[0, i], 1.0)[d[0, i]]
+            q = OP.softmax_t(z[0, i], 1.0)[d[0, i]]
+            u = uniform01(raw_words(5, STREAM_ACCEPT, step, 0, i, np.zeros(1, np.uint64)))[0]
+            assert abs(u * q - p) <= 1e-5 * max(p, q), (trial, a_o, a_g)
+            mism += 1
+            continue
+        take = int(out["n_emit"][0])
+        assert list(em_g[:take]) == em_o[:take], (trial, em_g, em_o)
+    assert mism <= 2
+
+
+def test_sampling_end_to_end_tiny():
+    """Level 2: sampling decode end to end; GPU and oracle decisions agree
+    wherever |u - p/q| > 1e-3 and draws agree where their Gumbel margins are
+    clear; the oracle follows the GPU's tokens."""
+    wl = S.WORKLOADS["tiny"].replace(sample=True, n_new=24)
+    P = Pair(wl)
+    seed = 11
+    P.prefill(seed)
+    K = wl.K
+    step = 1
+    checked = 0
+    while not P.oracle.all_done() and step < 40:
+        out = P.eng.alloc_step_outputs(want_logits=True)
+        P.eng.draft(out, True, 1.0, seed, step)
+        d_g = out["draft"].cpu().numpy()
+        z_g = out["draft_logits"].cpu().numpy()
+        d_o, z_o = P.oracle.draft(step, seed)
+        assert np.abs(z_g - z_o).max() <= LOGIT_TOL
+        P.eng.verify(out, None, 1.0)
+        y_g = out["logits"].cpu().numpy()
+        y_o = P.oracle.verify(d_g)
+        assert np.abs(y_g - y_o).max() <= LOGIT_TOL
+        P.eng.accept_commit(out, True, 1.0, seed, step)
+        a_g = int(out["accept_len"][0])
+        # decisions where clear
+        for i in range(min(a_g + 1, K)):
+            p = OP.softmax_t(y_o[0, i], 1.0)[d_g[0, i]]
+            q = OP.softmax_t(z_o[0, i], 1.0)[d_g[0, i]]
+            u = uniform01(raw_words(seed, STREAM_ACCEPT, step, 0, i, np.zeros(1, np.uint64)))[0]
+            if abs(u - p / q) > 1e-3:
+                assert (u * q < p) == (i < a_g), (step, i)
+                checked += 1
+        em = [int(x) for x in out["emitted"][0].cpu().numpy()[: a_g + 1]]
+        slots, _ = P.oracle.commit([a_g], [em if len(em) == a_g + 1 else em + [0] * (a_g + 1 - len(em))])
+        assert np.array_equal(out["kv_slots"][0].cpu().numpy()[: a_g + 1], slots[0][: a_g + 1])
+        step += 1
+    assert checked > 0
+    assert P.eng.last_status() == 0
+
+
+def test_state_errors_are_reported():
+    from paper_2504_18583_gb300 import pard
+    wl = S.WORKLOADS["tiny"]
+    P = Pair(wl)
+    out = P.eng.alloc_step_outputs()
+    with pytest.raises(pard.PardError) as e:
+        P.eng.draft(out)
+    assert e.value.code == -7
+    with pytest.raises(pard.PardError) as e:
+        P.eng.prefill([list(range(10))], 10_000, wl.K)
+    assert e.value.code == -1
