@@ -1,0 +1,387 @@
+"""Benchmark of the PARD decode step on GB300.
+
+Workload: LLaMA3.1-8B-shaped target with a LLaMA3.2-1B-shaped PARD draft
+(random-init bf16 weights drawn from a seed), batch 1, 512-token prompt,
+K = 8, greedy, 256 new tokens.  A step is one pass of the whole hot path:
+pard_draft + pard_verify + pard_accept_commit.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Prints one JSON line.  ``value`` is generated tokens/s with the weights and
+KV cache resident in HBM, timed with CUDA events over exactly K steps after
+W warm-up steps; ``roofline`` is the verify pass's algorithmic HBM bytes
+over its measured duration; ``e2e`` is the same metric for a full
+generation through the C ABI from a host prompt to host tokens; the CPU
+oracle is timed on the host cores on a bounded sample (``cpu_baseline``).
+``--impl reference`` times the CPU oracle itself, step for step.
+Under torchrun each rank runs an independent replica (the batch-1 step does
+not shard without tensor parallelism): value = all ranks' tokens / max time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "generated tokens/s (batch 1, 8B-shaped) + verify-step HBM GB/s as % of GB300 peak"
+WORKLOAD_DESC = ("LLaMA3.1-8B-shaped target (32 layers, d 4096, 32q/8kv heads, ffn 14336, vocab 128256) + "
+                 "LLaMA3.2-1B-shaped PARD draft (16 layers, d 2048), batch 1, 512-token prompt, K=8, greedy, "
+                 "256 new tokens, KV page 16")
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d.get("hbm_gbs", 6800.0), "measured"
+    return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"pard_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def verify_bytes(wl, ctx_tokens: float) -> float:
+    """Algorithmic HBM bytes of one verify pass: every target weight once
+    (layers, norms, LM head), the KV cache read over the context, the K+1
+    new rows' K/V written, and the logits statistics (not the logits, which
+    the greedy path does not store)."""
+    t = wl.target
+    kv_tok = t.kv_bytes_per_token()
+    w = t.streamed_weight_bytes()
+    rows = wl.K + 1
+    return w + ctx_tokens * kv_tok + rows * kv_tok
+
+
+def draft_bytes(wl, ctx_tokens: float) -> float:
+    d = wl.draft
+    return d.streamed_weight_bytes() + ctx_tokens * d.kv_bytes_per_token()
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (bounded sample)
+# ---------------------------------------------------------------------------
+def oracle_sample(wl, host_t, host_d, steps: int, prompt_len: int):
+    """Time `steps` oracle decode steps (draft + verify + accept + commit) of
+    the full-size models after a short prefill.  Returns (tokens/s, seconds
+    per step, threads)."""
+    import numpy as np
+    import oracle
+    swl = wl.replace(prompt_len=prompt_len, n_new=steps * (wl.K + 1) + 2)
+    dec = oracle.OracleDecoder(swl, host_t, host_d)
+    prompts = [p[:prompt_len] for p in wl.prompts()]
+    dec.prefill(prompts)
+    toks = 0
+    t0 = time.perf_counter()
+    for s in range(1, steps + 1):
+        d, z = dec.draft(s)
+        y = dec.verify(d)
+        acc, em = dec.accept(d, z, y, s)
+        _, nout = dec.commit(acc, em)
+        toks += sum(nout)
+    dt = time.perf_counter() - t0
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return toks / dt, dt / steps, threads
+
+
+def run_reference(args):
+    """--impl reference: the CPU oracle, step for step, on the host cores."""
+    import synthetic as S
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    wl = S.WORKLOADS["8b_greedy"]
+    host_t = S.model_weights(wl.target, wl.seed, S.TARGET)
+    host_d = S.model_weights(wl.draft, wl.seed, S.DRAFT)
+    import oracle
+    plen = 32
+    swl = wl.replace(prompt_len=plen, n_new=(args.steps + args.warmup) * (wl.K + 1) + 2)
+    dec = oracle.OracleDecoder(swl, host_t, host_d)
+    dec.prefill([p[:plen] for p in wl.prompts()])
+    for s in range(1, args.warmup + 1):
+        d, z = dec.draft(s)
+        y = dec.verify(d)
+        acc, em = dec.accept(d, z, y, s)
+        dec.commit(acc, em)
+    toks = 0
+    t0 = time.perf_counter()
+    for s in range(args.warmup + 1, args.warmup + args.steps + 1):
+        d, z = dec.draft(s)
+        y = dec.verify(d)
+        acc, em = dec.accept(d, z, y, s)
+        _, nout = dec.commit(acc, em)
+        toks += sum(nout)
+    dt = time.perf_counter() - t0
+    value = toks / dt
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    sample = (f"{args.steps} oracle decode steps (8B/1B full-size models, K=8) after a {plen}-token prefill "
+              "(the full 512-token prompt is ~8 TFLOP on the CPU)")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": "8b_greedy: " + WORKLOAD_DESC, "oracle_prompt_tokens": plen},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-steps", type=int, default=2)
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end generation (profiling runs)")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="profiling aid: truncate both models to this many layers (not a bench number)")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    args.warmup = max(args.warmup, 3)
+
+    import numpy as np
+    import torch
+    import synthetic as S
+    from paper_2504_18583_gb300 import _build, pard
+
+    ws, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    _build.build()
+
+    wl = S.WORKLOADS["8b_greedy"]
+    if args.layers:
+        wl = wl.replace(target=wl.target.replace(n_layers=args.layers),
+                        draft=wl.draft.replace(n_layers=min(args.layers, wl.draft.n_layers)))
+    if args.warmup + args.steps > wl.n_new - 2:
+        raise SystemExit("warmup + steps must stay below the generation length (256)")
+    keep_host = rank == 0 and not args.no_cpu_baseline
+    t_gen = time.perf_counter()
+    host_t = S.model_weights(wl.target, wl.seed, S.TARGET) if keep_host else None
+    host_d = S.model_weights(wl.draft, wl.seed, S.DRAFT) if keep_host else None
+    tw = S.device_weights(wl.target, wl.seed, S.TARGET, host=host_t)
+    dw = S.device_weights(wl.draft, wl.seed, S.DRAFT, host=host_d)
+    t_gen = time.perf_counter() - t_gen
+    prompts = [p.tolist() for p in wl.prompts()]
+    lens = [len(p) for p in prompts]
+    max_ctx = max(lens) + wl.n_new + 2 * wl.K + 16
+    eng = pard.PardEngine(wl.target, tw, wl.draft, dw, max_batch=wl.batch, max_k=wl.K, max_ctx=max_ctx,
+                          n_pages=wl.n_pages(), prefill_chunk=512, page_order_target=wl.page_order(S.TARGET),
+                          page_order_draft=wl.page_order(S.DRAFT))
+    stream = eng.stream
+
+    def generation(timed_steps: int, warmup: int, phase_events: bool):
+        eng.prefill(prompts, wl.n_new, wl.K)
+        out = eng.alloc_step_outputs()
+        for s in range(1, warmup + 1):
+            eng.step(out, step=s)
+        torch.cuda.synchronize()
+        if ws > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        ph = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(timed_steps)]
+        n_emit = torch.zeros(timed_steps, dtype=torch.int32, device="cuda")
+        launches = 0
+        ev[0].record(stream)
+        for i in range(timed_steps):
+            s = warmup + 1 + i
+            if phase_events:
+                ph[i][0].record(stream)
+            eng.draft(out, False, 1.0, 0, s)
+            launches += eng.launch_count()
+            if phase_events:
+                ph[i][1].record(stream)
+            eng.verify(out, None, 1.0)
+            launches += eng.launch_count()
+            if phase_events:
+                ph[i][2].record(stream)
+            eng.accept_commit(out, False, 1.0, 0, s)
+            launches += eng.launch_count()
+            if phase_events:
+                ph[i][3].record(stream)
+            n_emit[i:i + 1].copy_(out["n_emit"][:1])
+        ev[1].record(stream)
+        torch.cuda.synchronize()
+        ms = ev[0].elapsed_time(ev[1])
+        phases = None
+        if phase_events:
+            phases = {k: [ph[i][j].elapsed_time(ph[i][j + 1]) for i in range(timed_steps)]
+                      for j, k in enumerate(("draft", "verify", "accept"))}
+        return ms, int(n_emit.sum().item()), launches, phases
+
+    # untimed warm-up generation (JIT, caches)
+    generation(2, 3, False)
+    clocks = ClockSampler(local)
+    clocks.start()
+    ms, toks, launches, phases = generation(args.steps, args.warmup, True)
+    clk = clocks.stop()
+    n_state = eng.state()[0][0]
+    flags = eng.last_status()
+
+    # max over ranks
+    tot_toks = toks
+    ms_max = ms
+    if ws > 1:
+        t = torch.tensor([ms, float(toks)], dtype=torch.float64, device="cuda")
+        tmax = t.clone()
+        torch.distributed.all_reduce(tmax[:1], op=torch.distributed.ReduceOp.MAX)
+        torch.distributed.all_reduce(t[1:], op=torch.distributed.ReduceOp.SUM)
+        ms_max, tot_toks = float(tmax[0]), int(t[1])
+    value = tot_toks / (ms_max / 1e3)
+
+    # e2e: host prompt in (pinned), full generation, host tokens out each step
+    def e2e_run():
+        h_prompt = torch.tensor([t for p in prompts for t in p], dtype=torch.int32).pin_memory()
+        d_prompt = torch.empty_like(h_prompt, device="cuda")
+        h_out = torch.empty((wl.K + 1 + 1,), dtype=torch.int32).pin_memory()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        d_prompt.copy_(h_prompt, non_blocking=True)
+        first = torch.empty(wl.batch, dtype=torch.int32, device="cuda")
+        lens_c = (pard.ctypes.c_int32 * wl.batch)(*lens)
+        pard._check(pard.lib().pard_prefill(eng.ctx, d_prompt.data_ptr(), pard.ctypes.cast(lens_c, pard.ctypes.c_void_p),
+                                            wl.batch, wl.n_new, wl.K, 0, 1.0, 0, first.data_ptr(),
+                                            stream.cuda_stream), "pard_prefill")
+        eng.batch, eng.K = wl.batch, wl.K
+        out = eng.alloc_step_outputs()
+        gen = 1
+        steps = 0
+        while gen < wl.n_new:
+            steps += 1
+            eng.step(out, step=steps)
+            h_out[: wl.K + 1].copy_(out["emitted"][0], non_blocking=True)
+            h_out[wl.K + 1:].copy_(out["n_emit"][:1], non_blocking=True)
+            torch.cuda.current_stream().synchronize()
+            gen += int(h_out[wl.K + 1])
+        dt = time.perf_counter() - t0
+        return gen / dt, steps, h_prompt.numel() * 4
+
+    e2e_tps, e2e_steps, prompt_bytes = e2e_run() if not args.no_e2e else (None, 1, 0)
+
+    # roofline of the verify pass
+    peak, peak_kind = peaks()
+    ver_ms = statistics.median(phases["verify"])
+    dr_ms = statistics.median(phases["draft"])
+    acc_ms = statistics.median(phases["accept"])
+    ctx_mid = max(lens) + args.warmup + args.steps / 2.0  # mean context during the timed steps (a ~ 0)
+    vb = verify_bytes(wl, ctx_mid)
+    db = draft_bytes(wl, ctx_mid)
+    ver_gbs = vb / (ver_ms / 1e3) / 1e9
+    dr_gbs = db / (dr_ms / 1e3) / 1e9
+
+    cpu = None
+    if keep_host and ws == 1:
+        tps, sps, threads = oracle_sample(wl, host_t, host_d, args.cpu_steps, 32)
+        cpu = {"value": tps, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+               "sample": f"{args.cpu_steps} oracle decode steps of the full-size 8B/1B models after a 32-token "
+                         f"prefill ({sps:.2f} s per step)"}
+
+    alpha = 0.90  # acceptance the paper reports for PARD on LLaMA3.1-8B (Table 2, 4-alpha), context only
+    tok_per_step_proj = (1 - alpha ** (wl.K + 1)) / (1 - alpha)
+    step_ms = ms / args.steps
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights and prompt ids)",
+        "config": {"workload": "8b_greedy: " + WORKLOAD_DESC, "parallelism": f"replicas{ws}",
+                   "l2": "inputs larger than L2: 17.5 GB of weights stream from HBM every step",
+                   "acceptance": "random-init draft: ~0 candidates accepted, ~1 token per step"},
+        "roofline": {"bound": "hbm", "kernel": "verify pass (all its launches; GEMM-dominated)",
+                     "achieved": ver_gbs, "peak": peak, "unit": "GB/s", "frac": ver_gbs / peak,
+                     "peak_kind": peak_kind, "traffic": None, "bytes_per_launch": vb,
+                     "bytes_note": "target weights 15.01 GB + KV read over the context + K+1 rows of KV written"},
+        "phases_ms": {"draft": dr_ms, "verify": ver_ms, "accept": acc_ms},
+        "draft_roofline": {"achieved": dr_gbs, "frac": dr_gbs / peak, "bytes": db},
+        "projection": {"alpha": alpha, "tokens_per_step": tok_per_step_proj,
+                       "tokens_per_s": tok_per_step_proj / (step_ms / 1e3),
+                       "note": "acceptance rate from the paper (context); same measured step time"},
+        "e2e": None if args.no_e2e else {"value": e2e_tps, "unit": "tokens/s", "h2d_bytes_per_step": prompt_bytes / max(e2e_steps, 1),
+                "d2h_bytes_per_step": 4 * (wl.K + 2),
+                "note": "full generation through the C ABI: pinned host prompt in, prefill, every step's tokens out"},
+        "gpu_launches": launches,
+        "clocks": clk,
+        "cpu_baseline": cpu,
+        "device_status": flags,
+        "weights_gen_s": t_gen,
+        "final_n": n_state,
+    }
+    if args.layers:
+        line["config"]["profiling_layers"] = args.layers
+    if rank == 0:
+        print(json.dumps(line))
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())
