@@ -89,7 +89,15 @@ size_t pard_workspace_bytes(const pard_model_cfg* target, const pard_model_cfg* 
 size_t pard_kv_pool_bytes(const pard_model_cfg* target, const pard_model_cfg* draft, const pard_limits* lim);
 
 /* Validate shapes, record the borrowed pointers, carve the workspace and
- * build TMA descriptors and RoPE tables.  h_page_order_{target,draft}
+ * build TMA descriptors and RoPE tables.
+ * IN-PLACE PACKING: every projection and LM-head matrix whose row count is a
+ * multiple of 128 (64 for wg/wu) and whose column count is a multiple of 64
+ * is rearranged in place into 128-row x 64-column blocks (64-row for wg/wu),
+ * each stored contiguously with its 16-byte chunks rotated by (row mod 8), so
+ * that one weight tile is one contiguous 16 KB copy.  The bytes stay inside
+ * each matrix's own allocation; a matrix shared by both models is packed
+ * once.  pard_unpack_weights restores row-major order.  The embedding and
+ * the norm gains are never moved.  h_page_order_{target,draft}
  * (host, n_pages entries each, a permutation of 0..n_pages-1, or NULL for
  * the identity) give the order in which pages are handed to sequences.
  * Synchronises `stream` once (uploads tables).  On success *out owns host
@@ -165,6 +173,10 @@ pard_status pard_read_kv(pard_ctx* ctx, int32_t model, int32_t layer, int32_t b,
  * *h_flags (0 = clean); the word is cleared.  Returns PARD_ERR_TIMEOUT or
  * PARD_ERR_DEVICE_CHECK when bits are set. */
 pard_status pard_last_status(pard_ctx* ctx, uint32_t* h_flags, void* stream);
+
+/* Restore every matrix pard_load_weights packed to row-major order
+ * (synchronises `stream`).  The context accepts no further decode calls. */
+pard_status pard_unpack_weights(pard_ctx* ctx, void* stream);
 
 /* Kernel launches the last call enqueued (for launch accounting). */
 int32_t pard_launch_count(pard_ctx* ctx);

@@ -11,6 +11,7 @@
 #include <cstdio>
 #include <cstring>
 #include <mutex>
+#include <set>
 #include <string>
 #include <vector>
 
@@ -54,13 +55,14 @@ struct Model {
   const __nv_bfloat16* final_norm = nullptr;
   const __nv_bfloat16* lm_head = nullptr;
   std::vector<LayerW> L;
+  std::vector<LayerW> P;        // packed matrices (same pointers) or null where row-major
   std::vector<LayerMaps> maps;
   CUtensorMap lm_map;
+  const __nv_bfloat16* lm_pk = nullptr;
   __nv_bfloat16* kv = nullptr;  // [layer][K|V][page][hkv][ps][hd]
   size_t page_elems = 0;        // hkv * ps * hd
   int* page_table = nullptr;    // [max_batch][pt_ld]
   float2* rope = nullptr;       // [max_ctx][hd/2]
-  CUtensorMap xd_map[2], xo_map[2], xf_map[2], xg_map;  // [tt 16 | 64]
   int qd() const { return cfg.n_q_heads * cfg.head_dim; }
   int kvd() const { return cfg.n_kv_heads * cfg.head_dim; }
   __nv_bfloat16* kcache(int l) const { return kv + (size_t)(2 * l) * n_pages_ * page_elems; }
@@ -83,6 +85,7 @@ struct Dims {
   int m_dec;        // rows of a decode pass (B * 2K)
   int gcap;         // rows of the prefill LM-head input
   int dmax, qdmax, ffnmax, vocab, hkvmax, hdmax, w_tiles, pt_ld, sm;
+  int ffn_pad;      // widest FFN rounded up to whole 64-column blocks
   size_t attn_part_floats;
 };
 
@@ -92,10 +95,11 @@ Dims make_dims(const pard_model_cfg& t, const pard_model_cfg& d, const pard_limi
   Dims D;
   D.m_dec = lim.max_batch * 2 * lim.max_k;
   D.MC = round_up(std::max(D.m_dec, lim.prefill_chunk), 64);
-  D.gcap = round_up(std::max(lim.max_batch, 16), 16);
+  D.gcap = lim.max_batch <= 16 ? 16 : round_up(lim.max_batch, 64);  // whole token tiles of the LM-head input
   D.dmax = std::max(t.d_model, d.d_model);
   D.qdmax = std::max(t.n_q_heads * t.head_dim, d.n_q_heads * d.head_dim);
   D.ffnmax = std::max(t.ffn, d.ffn);
+  D.ffn_pad = round_up(D.ffnmax, 64);
   D.vocab = t.vocab;
   D.hkvmax = std::max(t.n_kv_heads, d.n_kv_heads);
   D.hdmax = std::max(t.head_dim, d.head_dim);
@@ -106,12 +110,14 @@ Dims make_dims(const pard_model_cfg& t, const pard_model_cfg& d, const pard_limi
   return D;
 }
 
+constexpr size_t kPackTmpBytes = (size_t)32 << 20;  // scratch for in-place weight packing
+
 struct WsOffsets {
   size_t h, xd, xo, xf, xg, ssq, ssqg, q, gpart, gcnt, apart, acnt, stats_t, stats_it, stats_d, stats_id, logits, dlogits;
   size_t row_tok, row_pos, row_seq, row_out, row_gi, seq_row0, m_dev;
   size_t g_row_seq, g_row_gi, g_m;
   size_t st_n, st_pc, st_pend, st_gen, st_max, st_done, st_d, st_dnorm, st_sa, st_snorm, st_spart, st_scnt;
-  size_t call, status, tmp_pos, pt[2], rope[2], g_plen;
+  size_t call, status, tmp_pos, pt[2], rope[2], g_plen, pack_tmp;
   size_t total;
 };
 
@@ -122,7 +128,7 @@ WsOffsets layout_ws(const Dims& D, const pard_limits& lim) {
   o.h = L.take((size_t)D.MC * D.dmax * 4);
   o.xd = L.take((size_t)2 * D.MC * D.dmax * 2);
   o.xo = L.take((size_t)2 * D.MC * D.qdmax * 2);
-  o.xf = L.take((size_t)2 * D.MC * D.ffnmax * 2);
+  o.xf = L.take((size_t)2 * D.MC * D.ffn_pad * 2);
   o.xg = L.take((size_t)2 * D.gcap * D.dmax * 2);
   o.ssq = L.take((size_t)(D.dmax / 128) * D.MC * 4);
   o.ssqg = L.take((size_t)(D.dmax / 128) * D.MC * 4);
@@ -165,6 +171,7 @@ WsOffsets layout_ws(const Dims& D, const pard_limits& lim) {
   for (int mi = 0; mi < 2; ++mi) o.pt[mi] = L.take((size_t)B * D.pt_ld * 4);
   for (int mi = 0; mi < 2; ++mi) o.rope[mi] = L.take((size_t)D.pt_ld * lim.page_size * (D.hdmax / 2) * 8);
   o.g_plen = L.take((size_t)B * 4);
+  o.pack_tmp = L.take(kPackTmpBytes);
   o.total = L.total + 256;
   return o;
 }
@@ -264,6 +271,9 @@ struct pard_ctx {
   int batch = 0, K = 0, n_new = 0;
   bool prefilled = false;
   bool last_draft_sampled = false;
+  bool unpacked = false;
+  std::vector<std::pair<__nv_bfloat16*, int>> packed_list;  // (matrix, R) packed in place, with N, K below
+  std::vector<std::pair<int, int>> packed_shape;
   int launches = 0;
 
   template <typename T>
@@ -313,7 +323,9 @@ void run_layers(pard_ctx* c, int mi, int rows_cap, int batch, int rows_per_seq, 
   const int row_blocks = (rows_per_seq + rb_rows - 1) / rb_rows;
   const int base = batch * cf.n_kv_heads * row_blocks;
   const int n_kt = (c->lim.max_ctx + 63) / 64;
-  int n_split = std::max(1, std::min(n_kt, (2 * c->sm + base - 1) / base));
+  // key splits: enough CTAs to cover the GPU, at least two 64-key tiles per split
+  int n_split = std::max(1, std::min(std::max(1, n_kt / 2), (2 * c->sm + base - 1) / base));
+  n_split = std::min(n_split, 32);  // the combine keeps 2 x 64 x n_split floats in the q buffer
   while (n_split > 1 && (size_t)base * n_split * 64 * (cf.head_dim + 2) > c->D.attn_part_floats) --n_split;
   if ((size_t)base * 64 * (cf.head_dim + 2) > c->D.attn_part_floats && n_split > 1) n_split = 1;
 
@@ -324,7 +336,8 @@ void run_layers(pard_ctx* c, int mi, int rows_cap, int batch, int rows_per_seq, 
     {
       GemmArgs a = gemm_base(c, rows_cap, tt);
       a.wmap[0] = Mp.q; a.wmap[1] = Mp.k; a.wmap[2] = Mp.v;
-      a.xmap = M.xd_map[ti];
+      a.wpk[0] = M.P[l].t[W_Q]; a.wpk[1] = M.P[l].t[W_K]; a.wpk[2] = M.P[l].t[W_V];
+      a.x = c->xd; a.x_rows = 2 * c->D.MC;
       a.nseg = 3;
       a.seg_tile0[0] = 0;
       a.seg_tile0[1] = qd / kTileN;
@@ -355,7 +368,7 @@ void run_layers(pard_ctx* c, int mi, int rows_cap, int batch, int rows_per_seq, 
       a.page_size = c->lim.page_size; a.n_pages = c->lim.n_pages;
       a.row_blocks = row_blocks; a.n_split = n_split;
       a.scale = (float)(1.0 / std::sqrt((double)cf.head_dim));
-      a.x_out = c->xo; a.x_ld = qd;
+      a.x_out = c->xo; a.x_rows = 2 * c->D.MC;
       a.part = c->apart; a.counters = c->acnt; a.status = c->status;
       launch_attention(a, base * n_split, s, true);
       c->launches++;
@@ -364,55 +377,60 @@ void run_layers(pard_ctx* c, int mi, int rows_cap, int batch, int rows_per_seq, 
     {
       GemmArgs a = gemm_base(c, rows_cap, tt);
       a.wmap[0] = Mp.o;
-      a.xmap = M.xo_map[ti];
+      a.wpk[0] = M.P[l].t[W_O];
+      a.x = c->xo; a.x_rows = 2 * c->D.MC;
       a.nseg = 1; a.seg_tile0[0] = 0; a.seg_tile0[1] = d / kTileN; a.seg_rows[0] = d;
       a.w_tiles = d / kTileN;
       a.kc = (qd + kChunkK - 1) / kChunkK;
       a.mode = MODE_RESID;
       a.h = c->h; a.h_ld = d; a.ssq_out = c->ssq;
-      a.x_next = c->xd; a.x_next_ld = d; a.g_next = W.t[W_MLP_NORM];
+      a.x_next = c->xd; a.g_next = W.t[W_MLP_NORM];
       run_gemm(c, a, tt, s);
     }
     // RMSNorm -> gate/up (paired 64-row tiles) -> SiLU(gate) * up
     {
       GemmArgs a = gemm_base(c, rows_cap, tt);
       a.wmap[0] = Mp.g; a.wmap[1] = Mp.u;
-      a.xmap = M.xd_map[ti];
+      a.wpk[0] = M.P[l].t[W_G]; a.wpk[1] = M.P[l].t[W_U];
+      if (!a.wpk[0] || !a.wpk[1]) a.wpk[0] = a.wpk[1] = nullptr;
+      a.x = c->xd; a.x_rows = 2 * c->D.MC;
       a.nseg = 1; a.pair = 1;
       a.w_tiles = (ffn + 63) / 64;
       a.seg_tile0[0] = 0; a.seg_tile0[1] = a.w_tiles; a.seg_rows[0] = ffn;
       a.kc = (d + kChunkK - 1) / kChunkK;
       a.mode = MODE_SWIGLU;
       a.ssq_in = c->ssq; a.ssq_tiles = d / 128; a.inv_d = 1.0f / d; a.eps = cf.rms_eps;
-      a.x_next = c->xf; a.x_next_ld = ffn;
+      a.x_next = c->xf;
       run_gemm(c, a, tt, s);
     }
     // down projection + residual; emits x = h * g_next (next layer's or the final norm)
     {
       GemmArgs a = gemm_base(c, rows_cap, tt);
       a.wmap[0] = Mp.dn;
-      a.xmap = M.xf_map[ti];
+      a.wpk[0] = M.P[l].t[W_D];
+      a.x = c->xf; a.x_rows = 2 * c->D.MC;
       a.nseg = 1; a.seg_tile0[0] = 0; a.seg_tile0[1] = d / kTileN; a.seg_rows[0] = d;
       a.w_tiles = d / kTileN;
       a.kc = (ffn + kChunkK - 1) / kChunkK;
       a.mode = MODE_RESID;
       a.h = c->h; a.h_ld = d; a.ssq_out = c->ssq;
-      a.x_next = c->xd; a.x_next_ld = d;
+      a.x_next = c->xd;
       a.g_next = l + 1 < cf.n_layers ? M.L[l + 1].t[W_ATTN_NORM] : M.final_norm;
       run_gemm(c, a, tt, s);
     }
   }
 }
 
-// LM head over the activation rows in xmap (final-norm scale from ssq_in).
-void run_lm_head(pard_ctx* c, int mi, const CUtensorMap& xmap, const float* ssq_in, int rows_cap, int tt,
+// LM head over the packed activation rows x (final-norm scale from ssq_in).
+void run_lm_head(pard_ctx* c, int mi, const __nv_bfloat16* x, int x_rows, const float* ssq_in, int rows_cap, int tt,
                  const int* m_dev, float* logits, const int* row_out, const int* row_gi, const int* row_seq,
                  float4* stats, int2* stats_i, int gumbel_stream, cudaStream_t s) {
   Model& M = c->m[mi];
   GemmArgs a = gemm_base(c, rows_cap, tt);
   a.m_dev = m_dev;
   a.wmap[0] = M.lm_map;
-  a.xmap = xmap;
+  a.wpk[0] = M.lm_pk;
+  a.x = x; a.x_rows = x_rows;
   a.nseg = 1;
   a.w_tiles = (M.cfg.vocab + kTileN - 1) / kTileN;
   a.seg_tile0[0] = 0; a.seg_tile0[1] = a.w_tiles; a.seg_rows[0] = M.cfg.vocab;
@@ -434,6 +452,19 @@ EmbedArgs embed_base(pard_ctx* c, int mi, int mode) {
   e.st = c->st; e.rp = c->rp;
   e.h = c->h; e.x = c->xd; e.ssq = c->ssq; e.m_cap = c->D.MC; e.status = c->status;
   return e;
+}
+
+// Move a [N][K] matrix between row-major order and the packed layout, one
+// batch of R-row blocks at a time through the workspace scratch.
+void pack_matrix(pard_ctx* c, __nv_bfloat16* w, int N, int K, int R, bool unpack, cudaStream_t s) {
+  const size_t block = (size_t)R * K;
+  const int per_batch = (int)std::max<size_t>(1, kPackTmpBytes / (block * 2));
+  __nv_bfloat16* tmp = c->template at<__nv_bfloat16>(c->o.pack_tmp);
+  for (int b0 = 0; b0 < N / R; b0 += per_batch) {
+    const int nb = std::min(per_batch, N / R - b0);
+    CK(cudaMemcpyAsync(tmp, w + (size_t)b0 * block, (size_t)nb * block * 2, cudaMemcpyDeviceToDevice, s));
+    launch_pack(tmp, w + (size_t)b0 * block, R, K, nb, unpack, s);
+  }
 }
 
 template <typename F>
@@ -551,11 +582,12 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
     CK(cudaMemsetAsync(c->status, 0, 4, s));
     CK(cudaMemsetAsync(c->xd, 0, (size_t)2 * c->D.MC * c->D.dmax * 2, s));
     CK(cudaMemsetAsync(c->xo, 0, (size_t)2 * c->D.MC * c->D.qdmax * 2, s));
-    CK(cudaMemsetAsync(c->xf, 0, (size_t)2 * c->D.MC * c->D.ffnmax * 2, s));
+    CK(cudaMemsetAsync(c->xf, 0, (size_t)2 * c->D.MC * c->D.ffn_pad * 2, s));
     CK(cudaMemsetAsync(c->xg, 0, (size_t)2 * c->D.gcap * c->D.dmax * 2, s));
 
     uint8_t* kvp = reinterpret_cast<uint8_t*>(kv_pool);
     std::vector<int> pt_init((size_t)lim->max_batch * c->D.pt_ld, -1);
+    std::set<const void*> packed_set;
     for (int mi = 0; mi < 2; ++mi) {
       Model& M = c->m[mi];
       M.cfg = *C[mi];
@@ -577,13 +609,35 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
         mp.dn = make_map(M.L[l].t[W_D], d, ffn, kTileN);
       }
       M.lm_map = make_map(M.lm_head, M.cfg.vocab, d, kTileN);
-      const int tts[2] = {16, 64};
-      for (int ti = 0; ti < 2; ++ti) {
-        M.xd_map[ti] = make_map(c->xd, 2 * c->D.MC, d, 2 * tts[ti]);
-        M.xo_map[ti] = make_map(c->xo, 2 * c->D.MC, qd, 2 * tts[ti]);
-        M.xf_map[ti] = make_map(c->xf, 2 * c->D.MC, ffn, 2 * tts[ti]);
+      // pack every matrix whose shape allows it, in place (each matrix once,
+      // also when the draft shares the target's tensors)
+      M.P.assign(M.cfg.n_layers, LayerW{});
+      auto pack = [&](const __nv_bfloat16* w, int N, int K, int R) -> const __nv_bfloat16* {
+        if (N % R || K % 64) return nullptr;
+        if (!packed_set.count(w)) {
+          pack_matrix(c, const_cast<__nv_bfloat16*>(w), N, K, R, false, s);
+          packed_set.insert(w);
+          c->packed_list.push_back({const_cast<__nv_bfloat16*>(w), R});
+          c->packed_shape.push_back({N, K});
+        }
+        return w;
+      };
+      for (int l = 0; l < M.cfg.n_layers; ++l) {
+        const LayerW& Wl = M.L[l];
+        LayerW& Pl = M.P[l];
+        for (int j = 0; j < 9; ++j) Pl.t[j] = nullptr;
+        Pl.t[W_Q] = pack(Wl.t[W_Q], qd, d, kTileN);
+        Pl.t[W_K] = pack(Wl.t[W_K], kvd, d, kTileN);
+        Pl.t[W_V] = pack(Wl.t[W_V], kvd, d, kTileN);
+        Pl.t[W_O] = pack(Wl.t[W_O], d, qd, kTileN);
+        if (ffn % 64 == 0 && d % 64 == 0) {
+          Pl.t[W_G] = pack(Wl.t[W_G], ffn, d, 64);
+          Pl.t[W_U] = pack(Wl.t[W_U], ffn, d, 64);
+        }
+        Pl.t[W_D] = pack(Wl.t[W_D], d, ffn, kTileN);
       }
-      M.xg_map = make_map(c->xg, 2 * c->D.gcap, d, 2 * pick_tt(c->D.gcap));
+      M.lm_pk = pack(M.lm_head, M.cfg.vocab, d, kTileN);
+      CK(cudaStreamSynchronize(s));
       M.kv = reinterpret_cast<__nv_bfloat16*>(kvp);
       M.n_pages_ = lim->n_pages;
       M.page_elems = (size_t)M.cfg.n_kv_heads * lim->page_size * M.cfg.head_dim;
@@ -623,6 +677,7 @@ pard_status pard_prefill(pard_ctx* c, const int32_t* d_tokens, const int32_t* h_
                          int32_t K, int32_t sample, float temperature, uint64_t seed, int32_t* d_first,
                          void* stream) {
   if (!c || !d_tokens || !h_lens || !d_first) return fail(PARD_ERR_ARG, "null argument");
+  if (c->unpacked) return fail(PARD_ERR_STATE, "weights were unpacked; load them again");
   if (batch < 1 || batch > c->lim.max_batch) return fail(PARD_ERR_ARG, "batch outside [1, max_batch]");
   if (K < 1 || K > c->lim.max_k) return fail(PARD_ERR_ARG, "K outside [1, max_k]");
   if (n_new < 1) return fail(PARD_ERR_ARG, "n_new < 1");
@@ -681,15 +736,15 @@ pard_status pard_prefill(pard_ctx* c, const int32_t* d_tokens, const int32_t* h_
           last_rows = rows;
         }
         if (mi == 0) {
-          launch_gather_rows(c->xd, M.cfg.d_model, c->ssq, M.cfg.d_model / 128, c->D.MC, last_rows - 1, c->xg,
-                             c->ssqg, c->D.MC, b, M.cfg.d_model, s, true);
+          launch_gather_rows(c->xd, 2 * c->D.MC, c->ssq, M.cfg.d_model / 128, c->D.MC, last_rows - 1, c->xg,
+                             2 * c->D.gcap, c->ssqg, c->D.MC, b, M.cfg.d_model, s, true);
           c->launches++;
         }
       }
       offset += len;
     }
     const int gtt = pick_tt(c->D.gcap);
-    run_lm_head(c, 0, c->m[0].xg_map, c->ssqg, batch, gtt, c->g_m, nullptr, nullptr, sample ? c->g_row_gi : nullptr,
+    run_lm_head(c, 0, c->xg, 2 * c->D.gcap, c->ssqg, batch, gtt, c->g_m, nullptr, nullptr, sample ? c->g_row_gi : nullptr,
                 c->g_row_seq, c->stats_t, c->stats_it, STREAM_BONUS, s);
     SelectArgs sa;
     std::memset(&sa, 0, sizeof(sa));
@@ -709,7 +764,7 @@ pard_status pard_prefill(pard_ctx* c, const int32_t* d_tokens, const int32_t* h_
 pard_status pard_draft(pard_ctx* c, int32_t sample, float temperature, uint64_t seed, uint64_t step, int32_t* d_out,
                        float* d_logits, void* stream) {
   if (!c) return fail(PARD_ERR_ARG, "null context");
-  if (!c->prefilled) return fail(PARD_ERR_STATE, "pard_draft before pard_prefill");
+  if (!c->prefilled) return fail(PARD_ERR_STATE, "pard_draft before pard_prefill (or after pard_unpack_weights)");
   if (sample && !(temperature > 0.f)) return fail(PARD_ERR_ARG, "temperature must be > 0 when sampling");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   c->launches = 0;
@@ -722,7 +777,7 @@ pard_status pard_draft(pard_ctx* c, int32_t sample, float temperature, uint64_t 
     Model& M = c->m[1];
     run_layers(c, 1, rows_cap, c->batch, 2 * c->K, M.page_table, s);
     const int tt = pick_tt(rows_cap);
-    run_lm_head(c, 1, M.xd_map[tt == 16 ? 0 : 1], c->ssq, rows_cap, tt, c->rp.m_dev,
+    run_lm_head(c, 1, c->xd, 2 * c->D.MC, c->ssq, rows_cap, tt, c->rp.m_dev,
                 (sample || d_logits) ? c->dlogits : nullptr, c->rp.row_out, c->rp.row_gi, c->rp.row_seq, c->stats_d,
                 c->stats_id, STREAM_DRAFT, s);
     SelectArgs sa;
@@ -763,7 +818,7 @@ pard_status pard_verify(pard_ctx* c, const int32_t* d_draft_in, float temperatur
     run_layers(c, 0, rows_cap, c->batch, c->K + 1, M.page_table, s);
     const int tt = pick_tt(rows_cap);
     const bool keep = c->last_draft_sampled || d_logits_out;
-    run_lm_head(c, 0, M.xd_map[tt == 16 ? 0 : 1], c->ssq, rows_cap, tt, c->rp.m_dev, keep ? c->logits : nullptr,
+    run_lm_head(c, 0, c->xd, 2 * c->D.MC, c->ssq, rows_cap, tt, c->rp.m_dev, keep ? c->logits : nullptr,
                 c->rp.row_out, nullptr, c->rp.row_seq, c->stats_t, c->stats_it, STREAM_BONUS, s);
     if (d_logits_out)
       CK(cudaMemcpyAsync(d_logits_out, c->logits, (size_t)c->batch * (c->K + 1) * c->D.vocab * 4,
@@ -877,6 +932,21 @@ pard_status pard_last_status(pard_ctx* c, uint32_t* h_flags, void* stream) {
     if (*h_flags & (ST_TIMEOUT_TMA | ST_TIMEOUT_MMA | ST_TIMEOUT_EPI))
       return fail(PARD_ERR_TIMEOUT, "a kernel pipeline wait ran out");
     if (*h_flags) return fail(PARD_ERR_DEVICE_CHECK, "a kernel flagged a bad index");
+    return PARD_OK;
+  });
+}
+
+pard_status pard_unpack_weights(pard_ctx* c, void* stream) {
+  if (!c) return fail(PARD_ERR_ARG, "null context");
+  if (c->unpacked) return PARD_OK;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return guarded([&]() -> pard_status {
+    for (size_t i = 0; i < c->packed_list.size(); ++i)
+      pack_matrix(c, c->packed_list[i].first, c->packed_shape[i].first, c->packed_shape[i].second,
+                  c->packed_list[i].second, true, s);
+    CK(cudaStreamSynchronize(s));
+    c->unpacked = true;
+    c->prefilled = false;
     return PARD_OK;
   });
 }

@@ -190,8 +190,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
     for (int d = 0; d < DPL; ++d) {
       __nv_bfloat16 hi, lo;
       split_bf16(val[d], hi, lo);
-      a.x_out[(size_t)(2 * m) * a.x_ld + col + d] = hi;
-      a.x_out[(size_t)(2 * m + 1) * a.x_ld + col + d] = lo;
+      a.x_out[xpk(2 * m, (int)col + d, a.x_rows)] = hi;
+      a.x_out[xpk(2 * m + 1, (int)col + d, a.x_rows)] = lo;
     }
   };
 
@@ -228,28 +228,45 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
   __syncthreads();
   if (!*sflag) return;
   __threadfence();
-#pragma unroll 1
-  for (int i = 0; i < QPW; ++i) {
-    const int qv = warp + 8 * i;
-    if (qv >= nqv) break;
+  // combine the splits in split order: w_s = exp(m_s - M) / sum_s l_s exp(m_s - M)
+  const int ns = a.n_split;
+  float* sw = sq;                       // [nqv][ns] weights (q is no longer needed)
+  float* sl = sq + kMaxQV * ns;         // [nqv][ns] split sums
+  for (int i = threadIdx.x; i < nqv * ns; i += kAttnThreads) {
+    const int qv = i / ns, s2 = i % ns;
+    const float* p = a.part + gbase + ((size_t)s2 * kMaxQV + qv) * (HD + 2);
+    sw[i] = __ldcg(p + HD);
+    sl[i] = __ldcg(p + HD + 1);
+  }
+  __syncthreads();
+  for (int qv = threadIdx.x; qv < nqv; qv += kAttnThreads) {
     float mx = -INFINITY;
-    for (int s = 0; s < a.n_split; ++s)
-      mx = fmaxf(mx, __ldcg(a.part + gbase + ((size_t)s * kMaxQV + qv) * (HD + 2) + HD));
-    float L = 0.f, acc[DPL];
-#pragma unroll
-    for (int d = 0; d < DPL; ++d) acc[d] = 0.f;
-    for (int s = 0; s < a.n_split; ++s) {
-      const float* p = a.part + gbase + ((size_t)s * kMaxQV + qv) * (HD + 2);
-      const float ms = __ldcg(p + HD);
-      if (ms == -INFINITY) continue;
-      const float w = expf(ms - mx);
-      L += __ldcg(p + HD + 1) * w;
-#pragma unroll
-      for (int d = 0; d < DPL; ++d) acc[d] += __ldcg(p + lane * DPL + d) * w;
+    for (int s2 = 0; s2 < ns; ++s2) mx = fmaxf(mx, sw[qv * ns + s2]);
+    float L = 0.f;
+    for (int s2 = 0; s2 < ns; ++s2) {
+      const float m2 = sw[qv * ns + s2];
+      const float w = m2 == -INFINITY ? 0.f : expf(m2 - mx);
+      sw[qv * ns + s2] = w;
+      L += sl[qv * ns + s2] * w;
     }
-#pragma unroll
-    for (int d = 0; d < DPL; ++d) acc[d] /= L;
-    write_out(qv, acc);
+    for (int s2 = 0; s2 < ns; ++s2) sw[qv * ns + s2] /= L;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < nqv * HD; i += kAttnThreads) {
+    const int qv = i / HD, d = i % HD;
+    float acc = 0.f;
+#pragma unroll 4
+    for (int s2 = 0; s2 < ns; ++s2) {
+      const float w = sw[qv * ns + s2];
+      if (w != 0.f) acc += __ldcg(a.part + gbase + ((size_t)s2 * kMaxQV + qv) * (HD + 2) + d) * w;
+    }
+    const int r = qv / GROUP, g = qv % GROUP;
+    const int m = row0 + r;
+    const size_t col = (size_t)(kvh * GROUP + g) * HD + d;
+    __nv_bfloat16 hi, lo;
+    split_bf16(acc, hi, lo);
+    a.x_out[xpk(2 * m, (int)col, a.x_rows)] = hi;
+    a.x_out[xpk(2 * m + 1, (int)col, a.x_rows)] = lo;
   }
   if (threadIdx.x == 0) a.counters[group_idx] = 0;
 }

@@ -110,6 +110,23 @@ __device__ __forceinline__ void tma_load_2d_hint(void* dst, const CUtensorMap* m
       : "memory");
 }
 
+// 1-D bulk copy of `bytes` contiguous bytes (16-byte aligned, multiple of 16)
+// into shared memory; completion is counted on bar.
+__device__ __forceinline__ void bulk_load_hint(void* dst, const void* src, uint32_t bytes, uint64_t* bar,
+                                               uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+
 // ---- tcgen05: tensor memory and UMMA ---------------------------------------
 __device__ __forceinline__ void tmem_alloc(uint32_t* smem_dst, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(smem_dst)),
@@ -173,6 +190,23 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t smem_addr) {
 // K-major, M x N tile.
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// ---- packed operand layouts -------------------------------------------------
+// Activations: a buffer of two_rows rows (hi/lo pairs) and K columns is stored
+// as 64-column blocks, [K/64][two_rows][64], each 128-byte row with its eight
+// 16-byte chunks rotated by (row mod 8) -- exactly the shared-memory image of a
+// 128-byte-swizzled K-major UMMA operand, so any 8-row-aligned run of rows of
+// one block is loaded with a single bulk copy.
+__host__ __device__ __forceinline__ size_t xpk(int r, int k, int two_rows) {
+  return ((size_t)(k >> 6) * two_rows + r) * 64 + (size_t)((((k & 63) >> 3) ^ (r & 7)) << 3) + (k & 7);
+}
+// Weights: a matrix [N][K] packed in blocks of R rows: [N/R][K/64][R][64], the
+// same 128-byte swizzle inside each R x 64 block (R = 128, or 64 for the
+// gate/up halves).
+__host__ __device__ __forceinline__ size_t wpk(int n, int k, int R, int K) {
+  const int b = n / R, r = n % R;
+  return (((size_t)b * (K >> 6) + (k >> 6)) * R + r) * 64 + (size_t)((((k & 63) >> 3) ^ (r & 7)) << 3) + (k & 7);
 }
 
 // ---- numerics --------------------------------------------------------------

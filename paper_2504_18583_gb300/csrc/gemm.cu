@@ -94,8 +94,8 @@ __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_tile, in
         *hp = hn;
         __nv_bfloat16 hi, lo;
         split_bf16(hn * g, hi, lo);
-        a.x_next[(size_t)(2 * m) * a.x_next_ld + n] = hi;
-        a.x_next[(size_t)(2 * m + 1) * a.x_next_ld + n] = lo;
+        a.x_next[xpk(2 * m, n, a.x_rows)] = hi;
+        a.x_next[xpk(2 * m + 1, n, a.x_rows)] = lo;
       }
       sq[j] = hn * hn;
     }
@@ -169,8 +169,8 @@ __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_tile, in
           const float gt = S.xch[j * kTileN + fr], up = S.xch[j * kTileN + 64 + fr];
           __nv_bfloat16 hi, lo;
           split_bf16(silu(gt) * up, hi, lo);
-          a.x_next[(size_t)(2 * m) * a.x_next_ld + n] = hi;
-          a.x_next[(size_t)(2 * m + 1) * a.x_next_ld + n] = lo;
+          a.x_next[xpk(2 * m, n, a.x_rows)] = hi;
+          a.x_next[xpk(2 * m + 1, n, a.x_rows)] = lo;
         }
       }
     }
@@ -303,48 +303,89 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
     // ---------------- TMA producer ----------------
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
-      for (int i = 0; i < a.nseg; ++i) tma_prefetch_desc(&a.wmap[i]);
-      if (a.pair) tma_prefetch_desc(&a.wmap[1]);
-      tma_prefetch_desc(&a.xmap);
-      const long n = u1 - u0;
-      const int npre = (int)(n < C::kStages ? n : C::kStages);
-      auto load_a = [&](long u, int s) {
-        const long t = u / a.kc;
-        const int kk = (int)(u % a.kc);
-        const int w_tile = (int)(t / a.tok_tiles);
-        uint8_t* dst = sA + s * C::kABytes;
+      for (int i = 0; i < kMaxSeg; ++i)
+        if ((i < a.nseg || (a.pair && i < 2)) && !a.wpk[i]) tma_prefetch_desc(&a.wmap[i]);
+      const int n = (int)(u1 - u0);
+      const int npre = n < C::kStages ? n : C::kStages;
+      // Unit cursor advanced incrementally: the producer issues one stage per
+      // wake-up with no divisions on the path between the 'empty' signal and
+      // the copies.
+      int kk = (int)(u0 % a.kc);
+      int w_tile = (int)((u0 / a.kc) / a.tok_tiles), tok_tile = (int)((u0 / a.kc) % a.tok_tiles);
+      const __nv_bfloat16* wsrc0 = nullptr;  // packed block base of the current weight tile (A)
+      const __nv_bfloat16* wsrc1 = nullptr;  // second half (gate/up pairs)
+      const CUtensorMap* wmap0 = nullptr;
+      int wrow = 0;                          // row-major fallback: first row of the tile
+      auto set_tile = [&]() {
         if (a.pair) {
-          tma_load_2d_hint(dst, &a.wmap[0], &full[s], kk * kChunkK, w_tile * 64, pol);
-          tma_load_2d_hint(dst + C::kABytes / 2, &a.wmap[1], &full[s], kk * kChunkK, w_tile * 64, pol);
+          if (a.wpk[0]) {
+            wsrc0 = a.wpk[0] + (size_t)w_tile * a.kc * 64 * 64;
+            wsrc1 = a.wpk[1] + (size_t)w_tile * a.kc * 64 * 64;
+          } else {
+            wsrc0 = wsrc1 = nullptr;
+            wrow = w_tile * 64;
+          }
         } else {
           const int seg = seg_of(a, w_tile);
-          tma_load_2d_hint(dst, &a.wmap[seg], &full[s], kk * kChunkK, (w_tile - a.seg_tile0[seg]) * kTileN, pol);
+          const int blk = w_tile - a.seg_tile0[seg];
+          wsrc0 = a.wpk[seg] ? a.wpk[seg] + (size_t)blk * a.kc * kTileN * 64 : nullptr;
+          wmap0 = &a.wmap[seg];
+          wrow = blk * kTileN;
         }
       };
-      auto load_b = [&](long u, int s) {
-        const long t = u / a.kc;
-        const int kk = (int)(u % a.kc);
-        const int tok_tile = (int)(t % a.tok_tiles);
-        tma_load_2d(sB + s * C::kBBytes, &a.xmap, &full[s], kk * kChunkK, tok_tile * 2 * TT);
+      set_tile();
+      const size_t x_tile_off = (size_t)2 * TT * 64;      // elements between token tiles of one block
+      const size_t x_blk = (size_t)a.x_rows * 64;         // elements between 64-column blocks
+      auto issue_a = [&](int s) {
+        uint8_t* dst = sA + s * C::kABytes;
+        if (a.pair) {
+          if (wsrc0) {
+            bulk_load_hint(dst, wsrc0 + (size_t)kk * 64 * 64, C::kABytes / 2, &full[s], pol);
+            bulk_load_hint(dst + C::kABytes / 2, wsrc1 + (size_t)kk * 64 * 64, C::kABytes / 2, &full[s], pol);
+          } else {
+            tma_load_2d_hint(dst, &a.wmap[0], &full[s], kk * kChunkK, wrow, pol);
+            tma_load_2d_hint(dst + C::kABytes / 2, &a.wmap[1], &full[s], kk * kChunkK, wrow, pol);
+          }
+        } else if (wsrc0) {
+          bulk_load_hint(dst, wsrc0 + (size_t)kk * kTileN * 64, C::kABytes, &full[s], pol);
+        } else {
+          tma_load_2d_hint(dst, wmap0, &full[s], kk * kChunkK, wrow, pol);
+        }
+      };
+      auto issue_b = [&](int s, int kk_, int tok_) {
+        bulk_load(sB + s * C::kBBytes, a.x + (size_t)kk_ * x_blk + (size_t)tok_ * x_tile_off, C::kBBytes, &full[s]);
+      };
+      auto advance = [&]() {
+        if (++kk == a.kc) {
+          kk = 0;
+          if (++tok_tile == a.tok_tiles) { tok_tile = 0; ++w_tile; }
+          set_tile();
+        }
       };
       // weights first: they do not depend on the previous kernel
+      int pre_kk[C::kStages], pre_tok[C::kStages];
       for (int i = 0; i < npre; ++i) {
         mbar_arrive_expect_tx(&full[i], C::kStageBytes);
-        load_a(u0 + i, i);
+        issue_a(i);
+        pre_kk[i] = kk;
+        pre_tok[i] = tok_tile;
+        advance();
       }
       pdl_wait();
-      for (int i = 0; i < npre; ++i) load_b(u0 + i, i);
-      for (long i = npre; i < n; ++i) {
-        const int s = (int)(i % C::kStages);
-        const uint32_t ph = (uint32_t)((i / C::kStages) & 1) ^ 1u;
+      for (int i = 0; i < npre; ++i) issue_b(i, pre_kk[i], pre_tok[i]);
+      int s = npre % C::kStages;
+      uint32_t ph = (uint32_t)((npre / C::kStages) & 1) ^ 1u;
+      for (int i = npre; i < n; ++i) {
         if (!mbar_wait(&empty[s], ph, abort_flag)) {
           set_status(a.status, ST_TIMEOUT_TMA);
           *abort_flag = 1;
           break;
         }
         mbar_arrive_expect_tx(&full[s], C::kStageBytes);
-        load_a(u0 + i, s);
-        load_b(u0 + i, s);
+        issue_a(s);
+        issue_b(s, kk, tok_tile);
+        advance();
+        if (++s == C::kStages) { s = 0; ph ^= 1u; }
       }
       pdl_trigger();
     }
@@ -402,15 +443,24 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       const int ab = seg_i % C::kNumAcc;
       const int w_tile = (int)(t / a.tok_tiles), tok_tile = (int)(t % a.tok_tiles);
       const int tok_base = tok_tile * TT;
-      if (a.ssq_in && et < TT) {
-        const int m = tok_base + et;
-        float r = 1.f;
-        if (m < M) {
-          float ss = 0.f;
-          for (int i = 0; i < a.ssq_tiles; ++i) ss += a.ssq_in[(size_t)i * a.m_cap + m];
-          r = 1.0f / sqrtf(ss * a.inv_d + a.eps);
+      if (a.ssq_in) {
+        // all partial sums of squares of this token tile in one round of loads,
+        // then a fixed-order sum per row (16 rows at a time through xch)
+        for (int c0 = 0; c0 < TT; c0 += kEpiTok) {
+          const int nld = a.ssq_tiles * kEpiTok;
+          for (int i = et; i < nld; i += 128) {
+            const int tile = i / kEpiTok, j = i % kEpiTok;
+            const int m = tok_base + c0 + j;
+            S.xch[i] = m < M ? __ldcg(a.ssq_in + (size_t)tile * a.m_cap + m) : 0.f;
+          }
+          epi_bar();
+          if (et < kEpiTok) {
+            float ss = 0.f;
+            for (int t2 = 0; t2 < a.ssq_tiles; ++t2) ss += S.xch[t2 * kEpiTok + et];
+            S.rs[c0 + et] = 1.0f / sqrtf(ss * a.inv_d + a.eps);
+          }
+          epi_bar();
         }
-        S.rs[et] = r;
       }
       if (!mbar_wait(&accf[ab], (uint32_t)((seg_i / C::kNumAcc) & 1), abort_flag)) {
         if (et == 0) set_status(a.status, ST_TIMEOUT_EPI);
@@ -438,9 +488,13 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
         for (int ch = 0; ch < C::kChunks; ++ch) {
           uint32_t r[32];
           tmem_ld32(tbase + ch * 32, r);
+          float4* dst = reinterpret_cast<float4*>(mine + ((size_t)ch * kTileN + fr) * kEpiTok);
 #pragma unroll
-          for (int j = 0; j < kEpiTok; ++j)
-            mine[(ch * kEpiTok + j) * kTileN + fr] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
+          for (int j4 = 0; j4 < 4; ++j4)
+            dst[j4] = make_float4(__uint_as_float(r[8 * j4 + 0]) + __uint_as_float(r[8 * j4 + 1]),
+                                  __uint_as_float(r[8 * j4 + 2]) + __uint_as_float(r[8 * j4 + 3]),
+                                  __uint_as_float(r[8 * j4 + 4]) + __uint_as_float(r[8 * j4 + 5]),
+                                  __uint_as_float(r[8 * j4 + 6]) + __uint_as_float(r[8 * j4 + 7]));
         }
         __threadfence();
         epi_bar();
@@ -459,15 +513,36 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
             float v[kEpiTok];
 #pragma unroll
             for (int j = 0; j < kEpiTok; ++j) v[j] = 0.f;
-            for (long cc = cf; cc <= cl; ++cc) {
-              if (cc == c) {
+            // contributors in CTA order, four partial tiles requested per round trip
+            for (long cc0 = cf; cc0 <= cl; cc0 += 4) {
+              float4 pv[4][4];
 #pragma unroll
-                for (int j = 0; j < kEpiTok; ++j) v[j] += __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
-              } else {
-                const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
-                const float* p = a.partials + ((size_t)cc * 2 + sl) * (kTileN * TT) + (ch * kEpiTok) * kTileN + fr;
+              for (int q4 = 0; q4 < 4; ++q4) {
+                const long cc = cc0 + q4;
+                if (cc <= cl && cc != c) {
+                  const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
+                  const float4* p = reinterpret_cast<const float4*>(
+                      a.partials + ((size_t)cc * 2 + sl) * (kTileN * TT) + ((size_t)ch * kTileN + fr) * kEpiTok);
 #pragma unroll
-                for (int j = 0; j < kEpiTok; ++j) v[j] += __ldcg(p + j * kTileN);
+                  for (int j4 = 0; j4 < 4; ++j4) pv[q4][j4] = __ldcg(p + j4);
+                }
+              }
+#pragma unroll
+              for (int q4 = 0; q4 < 4; ++q4) {
+                const long cc = cc0 + q4;
+                if (cc > cl) break;
+                if (cc == c) {
+#pragma unroll
+                  for (int j = 0; j < kEpiTok; ++j) v[j] += __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
+                } else {
+#pragma unroll
+                  for (int j4 = 0; j4 < 4; ++j4) {
+                    v[4 * j4 + 0] += pv[q4][j4].x;
+                    v[4 * j4 + 1] += pv[q4][j4].y;
+                    v[4 * j4 + 2] += pv[q4][j4].z;
+                    v[4 * j4 + 3] += pv[q4][j4].w;
+                  }
+                }
               }
             }
             epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S);

@@ -32,8 +32,11 @@ struct CallArgs {
 };
 
 struct GemmArgs {
-  CUtensorMap wmap[kMaxSeg];  // weights (A operand); pair mode: [0] gate, [1] up, 64-row boxes
-  CUtensorMap xmap;           // activations (B operand): row 2m = hi(m), 2m+1 = lo(m)
+  CUtensorMap wmap[kMaxSeg];  // row-major weights (A operand) for shapes that are not packed;
+                              // pair mode: [0] gate, [1] up, 64-row boxes
+  const __nv_bfloat16* wpk[kMaxSeg];  // packed weights (null: use wmap)
+  const __nv_bfloat16* x;     // packed activations (B operand): row 2m = hi(m), 2m+1 = lo(m)
+  int x_rows;                 // rows of the activation buffer (2 x row capacity)
   int nseg;
   int seg_tile0[kMaxSeg + 1]; // prefix sums of tiles per segment
   int seg_rows[kMaxSeg];      // rows of each segment
@@ -53,8 +56,7 @@ struct GemmArgs {
   float* h;
   int h_ld;
   float* ssq_out;
-  __nv_bfloat16* x_next;
-  int x_next_ld;
+  __nv_bfloat16* x_next;      // packed, x_rows rows
   const __nv_bfloat16* g_next;
   // MODE_QKV
   float* q_out;
@@ -93,8 +95,8 @@ struct AttnArgs {
   int row_blocks;             // row blocks per sequence (grid.y / ...)
   int n_split;                // key splits
   float scale;
-  __nv_bfloat16* x_out;       // [2*rows][hq*hd] hi/lo
-  int x_ld;
+  __nv_bfloat16* x_out;       // packed [2*rows][hq*hd] hi/lo
+  int x_rows;
   float* part;                // split partials
   int* counters;
   uint32_t* status;
@@ -140,7 +142,7 @@ struct EmbedArgs {
   DevState st;
   RowPlan rp;
   float* h;
-  __nv_bfloat16* x;
+  __nv_bfloat16* x;            // packed, 2 * m_cap rows
   float* ssq;
   int m_cap;
   uint32_t* status;
@@ -179,8 +181,10 @@ struct AcceptArgs {
 
 // launchers (gemm.cu, attention.cu, misc.cu)
 void launch_embed(const EmbedArgs& a, int grid, cudaStream_t s, bool pdl);
-void launch_gather_rows(const __nv_bfloat16* x, int x_ld, const float* ssq, int ssq_tiles, int m_cap_src, int src_row,
-                        __nv_bfloat16* xg, float* ssqg, int m_cap_dst, int dst_row, int d, cudaStream_t s, bool pdl);
+void launch_gather_rows(const __nv_bfloat16* x, int x_rows, const float* ssq, int ssq_tiles, int m_cap_src, int src_row,
+                        __nv_bfloat16* xg, int xg_rows, float* ssqg, int m_cap_dst, int dst_row, int d, cudaStream_t s,
+                        bool pdl);
+void launch_pack(const __nv_bfloat16* tmp, __nv_bfloat16* w, int R, int K, int nblocks, bool unpack, cudaStream_t s);
 void launch_select(const SelectArgs& a, cudaStream_t s, bool pdl);
 void launch_accept_greedy(const AcceptArgs& a, cudaStream_t s, bool pdl);
 void launch_accept_sample(const AcceptArgs& a, cudaStream_t s, bool pdl);

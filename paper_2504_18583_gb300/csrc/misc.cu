@@ -1,6 +1,7 @@
 // Small kernels of the decode step: row planning + embedding gather, the
 // draft's token selection from LM-head statistics, acceptance with KV
 // commit / rollback, and helpers for tests.
+#include <algorithm>
 #include <climits>
 
 #include "common.cuh"
@@ -104,8 +105,8 @@ __global__ void __launch_bounds__(128) embed_kernel(const __grid_constant__ Embe
       a.h[(size_t)m * a.d + c] = h;
       __nv_bfloat16 hi, lo;
       split_bf16(h * __bfloat162float(a.gain0[c]), hi, lo);
-      a.x[(size_t)(2 * m) * a.d + c] = hi;
-      a.x[(size_t)(2 * m + 1) * a.d + c] = lo;
+      a.x[xpk(2 * m, c, 2 * a.m_cap)] = hi;
+      a.x[xpk(2 * m + 1, c, 2 * a.m_cap)] = lo;
       ss += h * h;
     }
     ss = warp_sum(ss);
@@ -117,23 +118,54 @@ void launch_embed(const EmbedArgs& a, int grid, cudaStream_t s, bool pdl) {
   PARD_LAUNCH(embed_kernel, grid, 128, 0, s, pdl, a);
 }
 
-// Copy one activation row (hi/lo pair) and its sum-of-squares partials.
-__global__ void gather_rows_kernel(const __nv_bfloat16* x, int x_ld, const float* ssq, int ssq_tiles, int m_cap_src,
-                                   int src_row, __nv_bfloat16* xg, float* ssqg, int m_cap_dst, int dst_row, int d) {
+// Copy one activation row (hi/lo pair, packed layout) and its sum-of-squares partials.
+__global__ void gather_rows_kernel(const __nv_bfloat16* x, int x_rows, const float* ssq, int ssq_tiles, int m_cap_src,
+                                   int src_row, __nv_bfloat16* xg, int xg_rows, float* ssqg, int m_cap_dst, int dst_row,
+                                   int d) {
   pdl_wait();
   pdl_trigger();
   for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    xg[(size_t)(2 * dst_row) * d + c] = x[(size_t)(2 * src_row) * x_ld + c];
-    xg[(size_t)(2 * dst_row + 1) * d + c] = x[(size_t)(2 * src_row + 1) * x_ld + c];
+    xg[xpk(2 * dst_row, c, xg_rows)] = x[xpk(2 * src_row, c, x_rows)];
+    xg[xpk(2 * dst_row + 1, c, xg_rows)] = x[xpk(2 * src_row + 1, c, x_rows)];
   }
   for (int t = threadIdx.x; t < ssq_tiles; t += blockDim.x)
     ssqg[(size_t)t * m_cap_dst + dst_row] = ssq[(size_t)t * m_cap_src + src_row];
 }
 
-void launch_gather_rows(const __nv_bfloat16* x, int x_ld, const float* ssq, int ssq_tiles, int m_cap_src, int src_row,
-                        __nv_bfloat16* xg, float* ssqg, int m_cap_dst, int dst_row, int d, cudaStream_t s, bool pdl) {
-  PARD_LAUNCH(gather_rows_kernel, 1, 256, 0, s, pdl, x, x_ld, ssq, ssq_tiles, m_cap_src, src_row, xg, ssqg, m_cap_dst,
-              dst_row, d);
+void launch_gather_rows(const __nv_bfloat16* x, int x_rows, const float* ssq, int ssq_tiles, int m_cap_src, int src_row,
+                        __nv_bfloat16* xg, int xg_rows, float* ssqg, int m_cap_dst, int dst_row, int d, cudaStream_t s,
+                        bool pdl) {
+  PARD_LAUNCH(gather_rows_kernel, 1, 256, 0, s, pdl, x, x_rows, ssq, ssq_tiles, m_cap_src, src_row, xg, xg_rows, ssqg,
+              m_cap_dst, dst_row, d);
+}
+
+// Weight packing: nblocks consecutive R-row blocks of a [N][K] matrix move
+// between row-major order and the packed layout ([K/64][R][64] per block,
+// 16-byte chunks of row r rotated by r mod 8).  tmp holds a copy of the
+// blocks in the source order; w is overwritten in the destination order.
+__global__ void pack_kernel(const __nv_bfloat16* tmp, __nv_bfloat16* w, int R, int K, int nblocks, int unpack) {
+  const int kc = K / 64;
+  const size_t chunks = (size_t)nblocks * R * kc * 8;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < chunks; i += (size_t)gridDim.x * blockDim.x) {
+    const int j = (int)(i % 8);
+    size_t t = i / 8;
+    const int kk = (int)(t % kc);
+    t /= kc;
+    const int r = (int)(t % R);
+    const size_t b = t / R;
+    const size_t rm = (b * R + r) * (size_t)K + (size_t)kk * 64 + (size_t)j * 8;
+    const size_t pk = ((b * kc + kk) * R + r) * 64 + (size_t)((j ^ (r & 7)) << 3);
+    if (!unpack)
+      *reinterpret_cast<uint4*>(w + pk) = *reinterpret_cast<const uint4*>(tmp + rm);
+    else
+      *reinterpret_cast<uint4*>(w + rm) = *reinterpret_cast<const uint4*>(tmp + pk);
+  }
+}
+
+void launch_pack(const __nv_bfloat16* tmp, __nv_bfloat16* w, int R, int K, int nblocks, bool unpack, cudaStream_t s) {
+  const size_t chunks = (size_t)nblocks * R * (K / 64) * 8;
+  const int grid = (int)std::min<size_t>((chunks + 255) / 256, 4096);
+  PARD_LAUNCH(pack_kernel, grid, 256, 0, s, false, tmp, w, R, K, nblocks, unpack ? 1 : 0);
 }
 
 // ---------------------------------------------------------------------------

@@ -66,6 +66,8 @@ def lib() -> ctypes.CDLL:
         L.pard_get_state.argtypes = [vp, vp, vp, vp, vp]
         L.pard_read_kv.argtypes = [vp, i32, i32, i32, vp, i32, vp, vp, vp]
         L.pard_last_status.argtypes = [vp, P(ctypes.c_uint32), vp]
+        L.pard_unpack_weights.argtypes = [vp, vp]
+        L.pard_unpack_weights.restype = ctypes.c_int
         L.pard_launch_count.argtypes = [vp]
         L.pard_launch_count.restype = i32
         L.pard_last_error.argtypes = []
@@ -249,6 +251,10 @@ class PardEngine:
         if code not in (PARD_OK, -5, -6):
             _check(code, "pard_last_status")
         return flags.value
+
+    def unpack_weights(self) -> None:
+        """Restore the row-major weight layout (the engine is unusable after)."""
+        _check(lib().pard_unpack_weights(self.ctx, self.stream.cuda_stream), "pard_unpack_weights")
 
     def launch_count(self) -> int:
         return lib().pard_launch_count(self.ctx)

@@ -204,6 +204,27 @@ def test_sampling_end_to_end_tiny():
     assert P.eng.last_status() == 0
 
 
+def test_weight_packing_round_trip_restores_every_matrix():
+    """Loading packs the weight matrices in place; unpacking restores the
+    exact row-major bits (including a draft sharing the target's tensors)."""
+    import torch
+    wl = S.WORKLOADS["tiny"].replace(target=S.TARGET_8B.replace(n_layers=1, vocab=2048, mask_id=2047),
+                                     draft=S.DRAFT_1B.replace(n_layers=1, vocab=2048, mask_id=2047))
+    P = Pair(wl)
+    host = P.tw_host
+    dev = P.tw_dev
+    packed_any = not torch.equal(dev["layers"][0]["wq"].view(torch.int16).cpu(),
+                                 torch.from_numpy(host["layers"][0]["wq"].view("int16")))
+    assert packed_any, "wq should be in the packed layout while loaded"
+    P.eng.unpack_weights()
+    for name in ("wq", "wk", "wv", "wo", "wg", "wu", "wd"):
+        got = dev["layers"][0][name].view(torch.int16).cpu().numpy()
+        assert np.array_equal(got, host["layers"][0][name].view("int16")), name
+    assert np.array_equal(dev["lm_head"].view(torch.int16).cpu().numpy(), host["lm_head"].view("int16"))
+    with pytest.raises(Exception):
+        P.eng.prefill([[1, 2, 3]], 4, wl.K)
+
+
 def test_state_errors_are_reported():
     from paper_2504_18583_gb300 import pard
     wl = S.WORKLOADS["tiny"]
