@@ -106,7 +106,7 @@ Dims make_dims(const pard_model_cfg& t, const pard_model_cfg& d, const pard_limi
   D.w_tiles = (t.vocab + kTileN - 1) / kTileN;
   D.pt_ld = (lim.max_ctx + lim.page_size - 1) / lim.page_size;
   D.sm = sm;
-  D.attn_part_floats = (size_t)2048 * 64 * (D.hdmax + 2);
+  D.attn_part_floats = 0;  // splits combine through distributed shared memory
   return D;
 }
 
@@ -322,12 +322,12 @@ void run_layers(pard_ctx* c, int mi, int rows_cap, int batch, int rows_per_seq, 
   const int rb_rows = attention_rows_per_block(group);
   const int row_blocks = (rows_per_seq + rb_rows - 1) / rb_rows;
   const int base = batch * cf.n_kv_heads * row_blocks;
+  // key splits = CTAs per cluster (<= 8), enough to cover the GPU, at most
+  // one per 64-key chunk of the longest context
   const int n_kt = (c->lim.max_ctx + 63) / 64;
-  // key splits: enough CTAs to cover the GPU, at least two 64-key tiles per split
-  int n_split = std::max(1, std::min(std::max(1, n_kt / 2), (2 * c->sm + base - 1) / base));
-  n_split = std::min(n_split, 32);  // the combine keeps 2 x 64 x n_split floats in the q buffer
-  while (n_split > 1 && (size_t)base * n_split * 64 * (cf.head_dim + 2) > c->D.attn_part_floats) --n_split;
-  if ((size_t)base * 64 * (cf.head_dim + 2) > c->D.attn_part_floats && n_split > 1) n_split = 1;
+  const int n_split = std::max(1, std::min({8, n_kt, (2 * c->sm + base - 1) / base}));
+  (void)ti;
+  (void)tt;
 
   for (int l = 0; l < cf.n_layers; ++l) {
     const LayerW& W = M.L[l];
