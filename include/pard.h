@@ -178,6 +178,30 @@ pard_status pard_last_status(pard_ctx* ctx, uint32_t* h_flags, void* stream);
  * (synchronises `stream`).  The context accepts no further decode calls. */
 pard_status pard_unpack_weights(pard_ctx* ctx, void* stream);
 
+/* Acceptance from given logits, allocating nothing.  The paper has no
+ * counterpart: this is an interface for callers that cannot provide device
+ * memory of their own -- runtimes without a device allocator, or engines that
+ * plan all device memory ahead and forbid allocation on their serving path.
+ * Inputs and outputs are as for pard_set_logits + pard_accept_commit (the
+ * same kernels, same results): d_target_logits [batch][K+1][vocab],
+ * d_draft_logits [batch][K][vocab] (needed only when sample != 0), d_draft
+ * [batch][K]; outputs d_accept_len [batch] and d_emitted [batch][K+1] (-1
+ * after the emitted tokens).  Nothing is committed anywhere: no context is
+ * involved.
+ * Scratch: one fixed file-scope device array of about 6.3 MiB, sized for
+ * batch <= 16, 1 <= K <= 8, vocab <= 128256 (vocab a multiple of 8); larger
+ * sizes return PARD_ERR_ARG with a message.  Every GPU that loads the
+ * library keeps that array until the process exits.  The first call on a
+ * device looks up the array's device address (cudaGetSymbolAddress, with that
+ * device current) and caches it; make that first call before any stream
+ * capture.  All calls share the array and each call re-initialises the state
+ * it needs (including the counters that must start at zero), so calls whose
+ * work overlaps on the GPU race: issue them on one stream. */
+pard_status pard_accept_noalloc(const float* d_target_logits, const float* d_draft_logits, const int32_t* d_draft,
+                                int32_t batch, int32_t K, int32_t vocab, int32_t sample, float temperature,
+                                uint64_t seed, uint64_t step, int32_t* d_accept_len, int32_t* d_emitted,
+                                void* stream);
+
 /* Kernel launches the last call enqueued (for launch accounting). */
 int32_t pard_launch_count(pard_ctx* ctx);
 

@@ -33,6 +33,15 @@ struct CudaFail {
   cudaError_t e;
   const char* what;
 };
+
+}  // namespace
+
+// error message shared with the other translation units of the library
+namespace pard {
+void set_error(const std::string& msg) { g_err = msg; }
+}  // namespace pard
+
+namespace {
 #define CK(x)                                           \
   do {                                                  \
     cudaError_t e_ = (x);                               \

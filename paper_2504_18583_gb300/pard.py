@@ -66,6 +66,8 @@ def lib() -> ctypes.CDLL:
         L.pard_get_state.argtypes = [vp, vp, vp, vp, vp]
         L.pard_read_kv.argtypes = [vp, i32, i32, i32, vp, i32, vp, vp, vp]
         L.pard_last_status.argtypes = [vp, P(ctypes.c_uint32), vp]
+        L.pard_accept_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, f32, u64, u64, vp, vp, vp]
+        L.pard_accept_noalloc.restype = ctypes.c_int
         L.pard_unpack_weights.argtypes = [vp, vp]
         L.pard_unpack_weights.restype = ctypes.c_int
         L.pard_launch_count.argtypes = [vp]
