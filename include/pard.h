@@ -205,6 +205,21 @@ pard_status pard_accept_noalloc(const float* d_target_logits, const float* d_dra
 /* Kernel launches the last call enqueued (for launch accounting). */
 int32_t pard_launch_count(pard_ctx* ctx);
 
+/* Chooses how pard_draft / pard_verify run the forward pass (Sec. 3.1 draft
+ * pass, Sec. 3.2 verify pass).  enable = 1: a pass of at most 16
+ * rows (batch x 2K draft rows, batch x (K+1) verify rows) over fully packed
+ * weights, head_dim 64 or 128 and 2, 4 or 8 query heads per KV head runs as one
+ * persistent cooperative kernel (one CTA per SM) that streams every layer's
+ * weights and the LM head back to back; other passes, and every pass when the
+ * GPU cannot hold the cooperative grid, run one kernel per phase.  enable = 0
+ * (the default): always one kernel per phase.  Both compute the same results up to the order
+ * of floating-point sums.  Takes effect at the next pard_prefill.  Returns
+ * PARD_ERR_ARG for a null context. */
+pard_status pard_set_fused_pass(pard_ctx* ctx, int32_t enable);
+
+/* 1 when the last pard_draft or pard_verify ran the persistent kernel, else 0. */
+int32_t pard_fused_pass_used(pard_ctx* ctx);
+
 /* Thread-local message for the last failing call ("" if none). */
 const char* pard_last_error(void);
 

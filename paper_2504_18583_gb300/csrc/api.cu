@@ -95,6 +95,7 @@ struct Dims {
   int gcap;         // rows of the prefill LM-head input
   int dmax, qdmax, ffnmax, vocab, hkvmax, hdmax, w_tiles, pt_ld, sm;
   int ffn_pad;      // widest FFN rounded up to whole 64-column blocks
+  int fwd_phases;   // phase capacity of one persistent-pass table (5 per layer + LM head)
   size_t attn_part_floats;
 };
 
@@ -116,6 +117,7 @@ Dims make_dims(const pard_model_cfg& t, const pard_model_cfg& d, const pard_limi
   D.pt_ld = (lim.max_ctx + lim.page_size - 1) / lim.page_size;
   D.sm = sm;
   D.attn_part_floats = 0;  // splits combine through distributed shared memory
+  D.fwd_phases = 5 * std::max(t.n_layers, d.n_layers) + 1;
   return D;
 }
 
@@ -127,6 +129,7 @@ struct WsOffsets {
   size_t g_row_seq, g_row_gi, g_m;
   size_t st_n, st_pc, st_pend, st_gen, st_max, st_done, st_d, st_dnorm, st_sa, st_snorm, st_spart, st_scnt;
   size_t call, status, tmp_pos, pt[2], rope[2], g_plen, pack_tmp;
+  size_t fwd_tab, fwd_done, fwd_apart, fwd_acnt;
   size_t total;
 };
 
@@ -181,6 +184,12 @@ WsOffsets layout_ws(const Dims& D, const pard_limits& lim) {
   for (int mi = 0; mi < 2; ++mi) o.rope[mi] = L.take((size_t)D.pt_ld * lim.page_size * (D.hdmax / 2) * 8);
   o.g_plen = L.take((size_t)B * 4);
   o.pack_tmp = L.take(kPackTmpBytes);
+  // persistent pass: 4 phase tables ([model][logits kept]), their completion
+  // counters, and the attention split partials and arrival counters
+  o.fwd_tab = L.take((size_t)4 * D.fwd_phases * sizeof(Phase));
+  o.fwd_done = L.take((size_t)4 * D.fwd_phases * 4);
+  o.fwd_apart = L.take((size_t)kFwdMaxAttnItems * kMaxQVRows * (D.hdmax + 2) * 4);
+  o.fwd_acnt = L.take((size_t)kFwdMaxAttnItems * 4);
   o.total = L.total + 256;
   return o;
 }
@@ -284,6 +293,19 @@ struct pard_ctx {
   std::vector<std::pair<__nv_bfloat16*, int>> packed_list;  // (matrix, R) packed in place, with N, K below
   std::vector<std::pair<int, int>> packed_shape;
   int launches = 0;
+  // persistent pass, per [model][logits kept]: phase table in the workspace,
+  // its completion counters and how many passes it has run
+  struct FwdTable {
+    Phase* dev = nullptr;
+    unsigned* done = nullptr;
+    int n = 0;
+    unsigned passes = 0;
+    bool ok = false;
+  } fwd[2][2];
+  float* fwd_apart = nullptr;
+  int* fwd_acnt = nullptr;
+  bool fwd_enabled = false;  // persistent pass opt-in (pard_set_fused_pass)
+  bool fwd_used = false;  // the last draft / verify ran the persistent pass
 
   template <typename T>
   T* at(size_t off) { return reinterpret_cast<T*>(ws + off); }
@@ -317,123 +339,146 @@ void run_gemm(pard_ctx* c, GemmArgs& a, int tt, cudaStream_t s) {
   c->launches++;
 }
 
-// Decoder layers over the current row plan.  rows_cap: row capacity of the
-// pass; batch / rows_per_seq: attention work decomposition; pt_attn: page
-// table row base the attention kernel indexes by its sequence index.
-void run_layers(pard_ctx* c, int mi, int rows_cap, int batch, int rows_per_seq, const int* pt_attn,
-                cudaStream_t s) {
+// Attention work decomposition of a pass: row blocks per sequence, groups
+// (sequence x kv head x row block) and key splits (<= 8, enough CTAs to cover
+// the GPU, at most one per 64-key chunk of the longest context).
+struct AttnGeom {
+  int row_blocks, groups, n_split;
+};
+AttnGeom attn_geometry(pard_ctx* c, int mi, int rows_per_seq, int batch) {
+  const pard_model_cfg& cf = c->m[mi].cfg;
+  const int rb_rows = attention_rows_per_block(cf.n_q_heads / cf.n_kv_heads);
+  AttnGeom g;
+  g.row_blocks = (rows_per_seq + rb_rows - 1) / rb_rows;
+  g.groups = batch * cf.n_kv_heads * g.row_blocks;
+  const int n_kt = (c->lim.max_ctx + 63) / 64;
+  g.n_split = std::max(1, std::min({8, n_kt, (2 * c->sm + g.groups - 1) / g.groups}));
+  return g;
+}
+
+// Arguments of the five phases of layer l (QKV, attention, O, gate/up, down).
+struct LayerPlan {
+  GemmArgs qkv, o, gu, dn;
+  AttnArgs at;
+};
+LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch, const int* pt_attn,
+                     const AttnGeom& geo) {
   Model& M = c->m[mi];
   const pard_model_cfg& cf = M.cfg;
-  const int tt = pick_tt(rows_cap);
-  const int ti = tt == 16 ? 0 : 1;
   const int d = cf.d_model, qd = M.qd(), kvd = M.kvd(), ffn = cf.ffn;
-  const int group = cf.n_q_heads / cf.n_kv_heads;
-  const int rb_rows = attention_rows_per_block(group);
-  const int row_blocks = (rows_per_seq + rb_rows - 1) / rb_rows;
-  const int base = batch * cf.n_kv_heads * row_blocks;
-  // key splits = CTAs per cluster (<= 8), enough to cover the GPU, at most
-  // one per 64-key chunk of the longest context
-  const int n_kt = (c->lim.max_ctx + 63) / 64;
-  const int n_split = std::max(1, std::min({8, n_kt, (2 * c->sm + base - 1) / base}));
-  (void)ti;
-  (void)tt;
+  const LayerW& W = M.L[l];
+  const LayerMaps& Mp = M.maps[l];
+  LayerPlan P;
+  // fused RMSNorm -> QKV -> RoPE -> paged KV write
+  {
+    GemmArgs& a = P.qkv;
+    a = gemm_base(c, rows_cap, tt);
+    a.wmap[0] = Mp.q; a.wmap[1] = Mp.k; a.wmap[2] = Mp.v;
+    a.wpk[0] = M.P[l].t[W_Q]; a.wpk[1] = M.P[l].t[W_K]; a.wpk[2] = M.P[l].t[W_V];
+    a.x = c->xd; a.x_rows = 2 * c->D.MC;
+    a.nseg = 3;
+    a.seg_tile0[0] = 0;
+    a.seg_tile0[1] = qd / kTileN;
+    a.seg_tile0[2] = a.seg_tile0[1] + kvd / kTileN;
+    a.seg_tile0[3] = a.seg_tile0[2] + kvd / kTileN;
+    a.seg_rows[0] = qd; a.seg_rows[1] = kvd; a.seg_rows[2] = kvd;
+    a.w_tiles = a.seg_tile0[3];
+    a.kc = (d + kChunkK - 1) / kChunkK;
+    a.mode = MODE_QKV;
+    a.ssq_in = c->ssq; a.ssq_tiles = d / 128; a.inv_d = 1.0f / d; a.eps = cf.rms_eps;
+    a.q_out = c->q; a.q_ld = qd;
+    a.kcache = M.kcache(l); a.vcache = M.vcache(l);
+    a.page_table = M.page_table; a.pt_ld = c->D.pt_ld;
+    a.row_pos = c->rp.row_pos; a.row_seq = c->rp.row_seq;
+    a.rope = M.rope; a.hd = cf.head_dim; a.hkv = cf.n_kv_heads; a.page_size = c->lim.page_size;
+    a.n_pages = c->lim.n_pages;
+  }
+  // attention over the paged cache
+  {
+    AttnArgs& a = P.at;
+    std::memset(&a, 0, sizeof(a));
+    a.q = c->q; a.q_ld = qd;
+    a.kcache = M.kcache(l); a.vcache = M.vcache(l);
+    a.page_table = pt_attn; a.pt_ld = c->D.pt_ld;
+    a.row_pos = c->rp.row_pos; a.seq_row0 = c->rp.seq_row0; a.m_dev = c->rp.m_dev;
+    a.batch = batch; a.hq = cf.n_q_heads; a.hkv = cf.n_kv_heads; a.hd = cf.head_dim;
+    a.page_size = c->lim.page_size; a.n_pages = c->lim.n_pages;
+    a.row_blocks = geo.row_blocks; a.n_split = geo.n_split;
+    a.scale = (float)(1.0 / std::sqrt((double)cf.head_dim));
+    a.x_out = c->xo; a.x_rows = 2 * c->D.MC;
+    a.part = c->apart; a.counters = c->acnt; a.status = c->status;
+  }
+  // O projection + residual; emits x = h * g_mlp and the new row sums of squares
+  {
+    GemmArgs& a = P.o;
+    a = gemm_base(c, rows_cap, tt);
+    a.wmap[0] = Mp.o;
+    a.wpk[0] = M.P[l].t[W_O];
+    a.x = c->xo; a.x_rows = 2 * c->D.MC;
+    a.nseg = 1; a.seg_tile0[0] = 0; a.seg_tile0[1] = d / kTileN; a.seg_rows[0] = d;
+    a.w_tiles = d / kTileN;
+    a.kc = (qd + kChunkK - 1) / kChunkK;
+    a.mode = MODE_RESID;
+    a.h = c->h; a.h_ld = d; a.ssq_out = c->ssq;
+    a.x_next = c->xd; a.g_next = W.t[W_MLP_NORM];
+  }
+  // RMSNorm -> gate/up (paired 64-row tiles) -> SiLU(gate) * up
+  {
+    GemmArgs& a = P.gu;
+    a = gemm_base(c, rows_cap, tt);
+    a.wmap[0] = Mp.g; a.wmap[1] = Mp.u;
+    a.wpk[0] = M.P[l].t[W_G]; a.wpk[1] = M.P[l].t[W_U];
+    if (!a.wpk[0] || !a.wpk[1]) a.wpk[0] = a.wpk[1] = nullptr;
+    a.x = c->xd; a.x_rows = 2 * c->D.MC;
+    a.nseg = 1; a.pair = 1;
+    a.w_tiles = (ffn + 63) / 64;
+    a.seg_tile0[0] = 0; a.seg_tile0[1] = a.w_tiles; a.seg_rows[0] = ffn;
+    a.kc = (d + kChunkK - 1) / kChunkK;
+    a.mode = MODE_SWIGLU;
+    a.ssq_in = c->ssq; a.ssq_tiles = d / 128; a.inv_d = 1.0f / d; a.eps = cf.rms_eps;
+    a.x_next = c->xf;
+  }
+  // down projection + residual; emits x = h * g_next (next layer's or the final norm)
+  {
+    GemmArgs& a = P.dn;
+    a = gemm_base(c, rows_cap, tt);
+    a.wmap[0] = Mp.dn;
+    a.wpk[0] = M.P[l].t[W_D];
+    a.x = c->xf; a.x_rows = 2 * c->D.MC;
+    a.nseg = 1; a.seg_tile0[0] = 0; a.seg_tile0[1] = d / kTileN; a.seg_rows[0] = d;
+    a.w_tiles = d / kTileN;
+    a.kc = (ffn + kChunkK - 1) / kChunkK;
+    a.mode = MODE_RESID;
+    a.h = c->h; a.h_ld = d; a.ssq_out = c->ssq;
+    a.x_next = c->xd;
+    a.g_next = l + 1 < cf.n_layers ? M.L[l + 1].t[W_ATTN_NORM] : M.final_norm;
+  }
+  return P;
+}
 
-  for (int l = 0; l < cf.n_layers; ++l) {
-    const LayerW& W = M.L[l];
-    const LayerMaps& Mp = M.maps[l];
-    // fused RMSNorm -> QKV -> RoPE -> paged KV write
-    {
-      GemmArgs a = gemm_base(c, rows_cap, tt);
-      a.wmap[0] = Mp.q; a.wmap[1] = Mp.k; a.wmap[2] = Mp.v;
-      a.wpk[0] = M.P[l].t[W_Q]; a.wpk[1] = M.P[l].t[W_K]; a.wpk[2] = M.P[l].t[W_V];
-      a.x = c->xd; a.x_rows = 2 * c->D.MC;
-      a.nseg = 3;
-      a.seg_tile0[0] = 0;
-      a.seg_tile0[1] = qd / kTileN;
-      a.seg_tile0[2] = a.seg_tile0[1] + kvd / kTileN;
-      a.seg_tile0[3] = a.seg_tile0[2] + kvd / kTileN;
-      a.seg_rows[0] = qd; a.seg_rows[1] = kvd; a.seg_rows[2] = kvd;
-      a.w_tiles = a.seg_tile0[3];
-      a.kc = (d + kChunkK - 1) / kChunkK;
-      a.mode = MODE_QKV;
-      a.ssq_in = c->ssq; a.ssq_tiles = d / 128; a.inv_d = 1.0f / d; a.eps = cf.rms_eps;
-      a.q_out = c->q; a.q_ld = qd;
-      a.kcache = M.kcache(l); a.vcache = M.vcache(l);
-      a.page_table = M.page_table; a.pt_ld = c->D.pt_ld;
-      a.row_pos = c->rp.row_pos; a.row_seq = c->rp.row_seq;
-      a.rope = M.rope; a.hd = cf.head_dim; a.hkv = cf.n_kv_heads; a.page_size = c->lim.page_size;
-      a.n_pages = c->lim.n_pages;
-      run_gemm(c, a, tt, s);
-    }
-    // attention over the paged cache
-    {
-      AttnArgs a;
-      std::memset(&a, 0, sizeof(a));
-      a.q = c->q; a.q_ld = qd;
-      a.kcache = M.kcache(l); a.vcache = M.vcache(l);
-      a.page_table = pt_attn; a.pt_ld = c->D.pt_ld;
-      a.row_pos = c->rp.row_pos; a.seq_row0 = c->rp.seq_row0; a.m_dev = c->rp.m_dev;
-      a.batch = batch; a.hq = cf.n_q_heads; a.hkv = cf.n_kv_heads; a.hd = cf.head_dim;
-      a.page_size = c->lim.page_size; a.n_pages = c->lim.n_pages;
-      a.row_blocks = row_blocks; a.n_split = n_split;
-      a.scale = (float)(1.0 / std::sqrt((double)cf.head_dim));
-      a.x_out = c->xo; a.x_rows = 2 * c->D.MC;
-      a.part = c->apart; a.counters = c->acnt; a.status = c->status;
-      launch_attention(a, base * n_split, s, true);
-      c->launches++;
-    }
-    // O projection + residual; emits x = h * g_mlp and the new row sums of squares
-    {
-      GemmArgs a = gemm_base(c, rows_cap, tt);
-      a.wmap[0] = Mp.o;
-      a.wpk[0] = M.P[l].t[W_O];
-      a.x = c->xo; a.x_rows = 2 * c->D.MC;
-      a.nseg = 1; a.seg_tile0[0] = 0; a.seg_tile0[1] = d / kTileN; a.seg_rows[0] = d;
-      a.w_tiles = d / kTileN;
-      a.kc = (qd + kChunkK - 1) / kChunkK;
-      a.mode = MODE_RESID;
-      a.h = c->h; a.h_ld = d; a.ssq_out = c->ssq;
-      a.x_next = c->xd; a.g_next = W.t[W_MLP_NORM];
-      run_gemm(c, a, tt, s);
-    }
-    // RMSNorm -> gate/up (paired 64-row tiles) -> SiLU(gate) * up
-    {
-      GemmArgs a = gemm_base(c, rows_cap, tt);
-      a.wmap[0] = Mp.g; a.wmap[1] = Mp.u;
-      a.wpk[0] = M.P[l].t[W_G]; a.wpk[1] = M.P[l].t[W_U];
-      if (!a.wpk[0] || !a.wpk[1]) a.wpk[0] = a.wpk[1] = nullptr;
-      a.x = c->xd; a.x_rows = 2 * c->D.MC;
-      a.nseg = 1; a.pair = 1;
-      a.w_tiles = (ffn + 63) / 64;
-      a.seg_tile0[0] = 0; a.seg_tile0[1] = a.w_tiles; a.seg_rows[0] = ffn;
-      a.kc = (d + kChunkK - 1) / kChunkK;
-      a.mode = MODE_SWIGLU;
-      a.ssq_in = c->ssq; a.ssq_tiles = d / 128; a.inv_d = 1.0f / d; a.eps = cf.rms_eps;
-      a.x_next = c->xf;
-      run_gemm(c, a, tt, s);
-    }
-    // down projection + residual; emits x = h * g_next (next layer's or the final norm)
-    {
-      GemmArgs a = gemm_base(c, rows_cap, tt);
-      a.wmap[0] = Mp.dn;
-      a.wpk[0] = M.P[l].t[W_D];
-      a.x = c->xf; a.x_rows = 2 * c->D.MC;
-      a.nseg = 1; a.seg_tile0[0] = 0; a.seg_tile0[1] = d / kTileN; a.seg_rows[0] = d;
-      a.w_tiles = d / kTileN;
-      a.kc = (ffn + kChunkK - 1) / kChunkK;
-      a.mode = MODE_RESID;
-      a.h = c->h; a.h_ld = d; a.ssq_out = c->ssq;
-      a.x_next = c->xd;
-      a.g_next = l + 1 < cf.n_layers ? M.L[l + 1].t[W_ATTN_NORM] : M.final_norm;
-      run_gemm(c, a, tt, s);
-    }
+// Decoder layers over the current row plan, one launch per phase.
+// rows_cap: row capacity of the pass; batch / rows_per_seq: attention work
+// decomposition; pt_attn: page table row base the attention kernel indexes
+// by its sequence index.
+void run_layers(pard_ctx* c, int mi, int rows_cap, int batch, int rows_per_seq, const int* pt_attn,
+                cudaStream_t s) {
+  const int tt = pick_tt(rows_cap);
+  const AttnGeom geo = attn_geometry(c, mi, rows_per_seq, batch);
+  for (int l = 0; l < c->m[mi].cfg.n_layers; ++l) {
+    LayerPlan P = layer_plan(c, mi, l, rows_cap, tt, batch, pt_attn, geo);
+    run_gemm(c, P.qkv, tt, s);
+    launch_attention(P.at, geo.groups * geo.n_split, s, true);
+    c->launches++;
+    run_gemm(c, P.o, tt, s);
+    run_gemm(c, P.gu, tt, s);
+    run_gemm(c, P.dn, tt, s);
   }
 }
 
 // LM head over the packed activation rows x (final-norm scale from ssq_in).
-void run_lm_head(pard_ctx* c, int mi, const __nv_bfloat16* x, int x_rows, const float* ssq_in, int rows_cap, int tt,
+GemmArgs lm_args(pard_ctx* c, int mi, const __nv_bfloat16* x, int x_rows, const float* ssq_in, int rows_cap, int tt,
                  const int* m_dev, float* logits, const int* row_out, const int* row_gi, const int* row_seq,
-                 float4* stats, int2* stats_i, int gumbel_stream, cudaStream_t s) {
+                 float4* stats, int2* stats_i, int gumbel_stream) {
   Model& M = c->m[mi];
   GemmArgs a = gemm_base(c, rows_cap, tt);
   a.m_dev = m_dev;
@@ -448,7 +493,124 @@ void run_lm_head(pard_ctx* c, int mi, const __nv_bfloat16* x, int x_rows, const 
   a.ssq_in = ssq_in; a.ssq_tiles = M.cfg.d_model / 128; a.inv_d = 1.0f / M.cfg.d_model; a.eps = M.cfg.rms_eps;
   a.logits = logits; a.row_out = row_out; a.row_gi = row_gi; a.row_seq = row_seq;
   a.stats = stats; a.stats_i = stats_i; a.vocab = M.cfg.vocab; a.gumbel_stream = gumbel_stream;
+  return a;
+}
+
+void run_lm_head(pard_ctx* c, int mi, const __nv_bfloat16* x, int x_rows, const float* ssq_in, int rows_cap, int tt,
+                 const int* m_dev, float* logits, const int* row_out, const int* row_gi, const int* row_seq,
+                 float4* stats, int2* stats_i, int gumbel_stream, cudaStream_t s) {
+  GemmArgs a = lm_args(c, mi, x, x_rows, ssq_in, rows_cap, tt, m_dev, logits, row_out, row_gi, row_seq, stats, stats_i,
+                       gumbel_stream);
   run_gemm(c, a, tt, s);
+}
+
+// ---------------------------------------------------------------------------
+// Persistent pass: the phase table of one decode forward (draft or verify),
+// run by one cooperative launch of fwd_kernel instead of 5 launches per layer
+// plus the LM head.  It covers passes of <= 16 rows over fully packed weights
+// with head shapes the kernel is instantiated for; everything else (prefill,
+// larger batches) takes the per-phase kernels.
+// ---------------------------------------------------------------------------
+bool fwd_shape_ok(const Model& M) {
+  const int hd = M.cfg.head_dim, group = M.cfg.n_q_heads / M.cfg.n_kv_heads;
+  if (!((hd == 128 || hd == 64) && (group == 2 || group == 4 || group == 8))) return false;
+  if (!M.lm_pk) return false;
+  for (int l = 0; l < M.cfg.n_layers; ++l)
+    for (int w : {W_Q, W_K, W_V, W_O, W_G, W_U, W_D})
+      if (!M.P[l].t[w]) return false;
+  return true;
+}
+
+// Builds (on the host) and uploads the phase table of model mi for the
+// current batch and K.  keep: the LM head also writes full logits.
+void build_fwd(pard_ctx* c, int mi, int keep, cudaStream_t s) {
+  pard_ctx::FwdTable& T = c->fwd[mi][keep];
+  T.ok = false;
+  T.n = 0;
+  T.passes = 0;
+  Model& M = c->m[mi];
+  const bool draft = mi == 1;
+  const int rows_per_seq = draft ? 2 * c->K : c->K + 1;
+  const int rows_cap = c->batch * rows_per_seq;
+  if (!c->fwd_enabled || rows_cap > kFwdTT || !fwd_shape_ok(M)) return;
+  if (5 * M.cfg.n_layers + 1 > c->D.fwd_phases) return;
+  AttnGeom geo = attn_geometry(c, mi, rows_per_seq, c->batch);
+  // one CTA per SM runs the attention items (group, split) = c, c + grid, ...
+  const int n_kt = (c->lim.max_ctx + 63) / 64;
+  geo.n_split = std::max(1, std::min({kFwdMaxSplit, n_kt, c->sm / std::max(1, geo.groups)}));
+  if (geo.groups * geo.n_split > kFwdMaxAttnItems) return;
+  std::vector<Phase> ph;
+  ph.reserve(5 * M.cfg.n_layers + 1);
+  auto gemm_phase = [&](const GemmArgs& g, int dep) {
+    Phase p;
+    std::memset(&p, 0, sizeof(p));
+    p.type = PH_GEMM;
+    p.dep = dep;
+    p.g = g;
+    ph.push_back(p);
+  };
+  for (int l = 0; l < M.cfg.n_layers; ++l) {
+    LayerPlan P = layer_plan(c, mi, l, rows_cap, kFwdTT, c->batch, M.page_table, geo);
+    const int prev = (int)ph.size() - 1;  // -1 for the first layer: the embedding kernel precedes the launch
+    gemm_phase(P.qkv, prev);
+    Phase a;
+    std::memset(&a, 0, sizeof(a));
+    a.type = PH_ATTN;
+    a.dep = (int)ph.size() - 1;
+    a.attn_groups = geo.groups;
+    a.attn_split = geo.n_split;
+    a.at = P.at;
+    ph.push_back(a);
+    gemm_phase(P.o, (int)ph.size() - 1);
+    gemm_phase(P.gu, (int)ph.size() - 1);
+    gemm_phase(P.dn, (int)ph.size() - 1);
+  }
+  GemmArgs lm = draft ? lm_args(c, 1, c->xd, 2 * c->D.MC, c->ssq, rows_cap, kFwdTT, c->rp.m_dev,
+                                keep ? c->dlogits : nullptr, c->rp.row_out, c->rp.row_gi, c->rp.row_seq, c->stats_d,
+                                c->stats_id, STREAM_DRAFT)
+                      : lm_args(c, 0, c->xd, 2 * c->D.MC, c->ssq, rows_cap, kFwdTT, c->rp.m_dev,
+                                keep ? c->logits : nullptr, c->rp.row_out, nullptr, c->rp.row_seq, c->stats_t,
+                                c->stats_it, STREAM_BONUS);
+  gemm_phase(lm, (int)ph.size() - 1);
+  for (const Phase& p : ph)
+    if (p.type == PH_GEMM && p.g.tok_tiles != 1) return;
+  CK(cudaMemcpyAsync(T.dev, ph.data(), ph.size() * sizeof(Phase), cudaMemcpyHostToDevice, s));
+  CK(cudaMemsetAsync(T.done, 0, ph.size() * 4, s));
+  CK(cudaStreamSynchronize(s));
+  T.n = (int)ph.size();
+  T.ok = true;
+}
+
+// Runs the persistent pass of model mi if its table is usable; false means
+// the caller runs the per-phase kernels instead.
+bool try_fwd(pard_ctx* c, int mi, int keep, cudaStream_t s) {
+  pard_ctx::FwdTable& T = c->fwd[mi][keep];
+  c->fwd_used = false;
+  if (!c->fwd_enabled || !T.ok) return false;
+  FwdArgs f;
+  std::memset(&f, 0, sizeof(f));
+  f.phases = T.dev;
+  f.n_phases = T.n;
+  f.done = T.done;
+  f.target = (T.passes + 1) * (unsigned)c->sm;
+  f.attn_part = c->fwd_apart;
+  f.attn_cnt = c->fwd_acnt;
+  f.status = c->status;
+  f.m_dev = c->rp.m_dev;
+  f.m_cap = c->D.MC;
+  const Model& M = c->m[mi];
+  cudaError_t e = launch_fwd(f, M.cfg.head_dim, M.cfg.n_q_heads / M.cfg.n_kv_heads, c->sm, s);
+  if (e != cudaSuccess) {
+    // not launchable here (e.g. the grid cannot be co-resident): per-phase kernels from now on
+    (void)cudaGetLastError();
+    for (auto& row : c->fwd)
+      for (auto& t : row) t.ok = false;
+    return false;
+  }
+  T.passes++;
+  c->launches++;
+  c->fwd_used = true;
+  return true;
 }
 
 EmbedArgs embed_base(pard_ctx* c, int mi, int mode) {
@@ -583,10 +745,19 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
     c->st.samp_cnt = c->at<int>(o.st_scnt); c->st.kmax = lim->max_k;
     c->call = c->at<CallArgs>(o.call); c->status = c->at<uint32_t>(o.status);
     c->tmp_pos = c->at<int>(o.tmp_pos); c->g_plen = c->at<int>(o.g_plen);
+    for (int mi = 0; mi < 2; ++mi)
+      for (int kl = 0; kl < 2; ++kl) {
+        const size_t t = (size_t)(2 * mi + kl) * c->D.fwd_phases;
+        c->fwd[mi][kl].dev = c->at<Phase>(o.fwd_tab) + t;
+        c->fwd[mi][kl].done = c->at<unsigned>(o.fwd_done) + t;
+      }
+    c->fwd_apart = c->at<float>(o.fwd_apart);
+    c->fwd_acnt = c->at<int>(o.fwd_acnt);
 
     // counters start at zero; the reduction kernels leave them at zero
     CK(cudaMemsetAsync(c->gcnt, 0, 65536 * 4, s));
     CK(cudaMemsetAsync(c->acnt, 0, 65536 * 4, s));
+    CK(cudaMemsetAsync(c->fwd_acnt, 0, (size_t)kFwdMaxAttnItems * 4, s));
     CK(cudaMemsetAsync(c->st.samp_cnt, 0, lim->max_batch * 4, s));
     CK(cudaMemsetAsync(c->status, 0, 4, s));
     CK(cudaMemsetAsync(c->xd, 0, (size_t)2 * c->D.MC * c->D.dmax * 2, s));
@@ -763,6 +934,8 @@ pard_status pard_prefill(pard_ctx* c, const int32_t* d_tokens, const int32_t* h_
     sa.out = d_first; sa.plen = c->g_plen; sa.n_new = n_new;
     launch_select(sa, s, true);
     c->launches++;
+    for (int mi = 0; mi < 2; ++mi)
+      for (int keep = 0; keep < 2; ++keep) build_fwd(c, mi, keep, s);
     CK(cudaStreamSynchronize(s));
     CK(cudaGetLastError());
     c->prefilled = true;
@@ -784,11 +957,13 @@ pard_status pard_draft(pard_ctx* c, int32_t sample, float temperature, uint64_t 
     launch_embed(e, rows_cap, s, true);
     c->launches++;
     Model& M = c->m[1];
-    run_layers(c, 1, rows_cap, c->batch, 2 * c->K, M.page_table, s);
-    const int tt = pick_tt(rows_cap);
-    run_lm_head(c, 1, c->xd, 2 * c->D.MC, c->ssq, rows_cap, tt, c->rp.m_dev,
-                (sample || d_logits) ? c->dlogits : nullptr, c->rp.row_out, c->rp.row_gi, c->rp.row_seq, c->stats_d,
-                c->stats_id, STREAM_DRAFT, s);
+    const int keep = (sample || d_logits) ? 1 : 0;
+    if (!try_fwd(c, 1, keep, s)) {
+      run_layers(c, 1, rows_cap, c->batch, 2 * c->K, M.page_table, s);
+      const int tt = pick_tt(rows_cap);
+      run_lm_head(c, 1, c->xd, 2 * c->D.MC, c->ssq, rows_cap, tt, c->rp.m_dev, keep ? c->dlogits : nullptr,
+                  c->rp.row_out, c->rp.row_gi, c->rp.row_seq, c->stats_d, c->stats_id, STREAM_DRAFT, s);
+    }
     SelectArgs sa;
     std::memset(&sa, 0, sizeof(sa));
     sa.mode = SEL_DRAFT;
@@ -824,11 +999,13 @@ pard_status pard_verify(pard_ctx* c, const int32_t* d_draft_in, float temperatur
     launch_embed(e, rows_cap, s, true);
     c->launches++;
     Model& M = c->m[0];
-    run_layers(c, 0, rows_cap, c->batch, c->K + 1, M.page_table, s);
-    const int tt = pick_tt(rows_cap);
-    const bool keep = c->last_draft_sampled || d_logits_out;
-    run_lm_head(c, 0, c->xd, 2 * c->D.MC, c->ssq, rows_cap, tt, c->rp.m_dev, keep ? c->logits : nullptr,
-                c->rp.row_out, nullptr, c->rp.row_seq, c->stats_t, c->stats_it, STREAM_BONUS, s);
+    const int keep = (c->last_draft_sampled || d_logits_out) ? 1 : 0;
+    if (!try_fwd(c, 0, keep, s)) {
+      run_layers(c, 0, rows_cap, c->batch, c->K + 1, M.page_table, s);
+      const int tt = pick_tt(rows_cap);
+      run_lm_head(c, 0, c->xd, 2 * c->D.MC, c->ssq, rows_cap, tt, c->rp.m_dev, keep ? c->logits : nullptr,
+                  c->rp.row_out, nullptr, c->rp.row_seq, c->stats_t, c->stats_it, STREAM_BONUS, s);
+    }
     if (d_logits_out)
       CK(cudaMemcpyAsync(d_logits_out, c->logits, (size_t)c->batch * (c->K + 1) * c->D.vocab * 4,
                          cudaMemcpyDeviceToDevice, s));
@@ -961,6 +1138,17 @@ pard_status pard_unpack_weights(pard_ctx* c, void* stream) {
 }
 
 int32_t pard_launch_count(pard_ctx* c) { return c ? c->launches : 0; }
+
+pard_status pard_set_fused_pass(pard_ctx* c, int32_t enable) {
+  if (!c) return fail(PARD_ERR_ARG, "null context");
+  c->fwd_enabled = enable != 0;
+  if (!c->fwd_enabled)
+    for (auto& row : c->fwd)
+      for (auto& t : row) t.ok = false;
+  return PARD_OK;
+}
+
+int32_t pard_fused_pass_used(pard_ctx* c) { return c && c->fwd_used ? 1 : 0; }
 
 void pard_destroy(pard_ctx* c) { delete c; }
 

@@ -1,0 +1,310 @@
+// Shared device code of the paged multi-query-position GQA attention: the
+// per-(sequence, kv head, row block) partial over a range of 32-key chunks on
+// the tensor cores.  Included by the cluster attention kernel (attention.cu)
+// and the persistent decode kernel (fwd_kernel.cuh).
+#pragma once
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace pard {
+
+constexpr int kAttnThreads = 128;  // 4 warps x 16 query vectors
+constexpr int kMaxQV = kMaxQVRows;
+constexpr int kKeyChunk = 32;
+constexpr int kMaxCluster = 8;
+constexpr int kAttnPageCache = 512;  // page ids of one work unit's key range held in shared memory
+
+// Shared memory of one work unit: K and V chunks double-buffered, Q as bf16
+// hi and lo rows (the MMA A operand, read with ldmatrix), then the page id
+// cache; the partial result (o, m, l) reuses the front at the end.
+template <int HD>
+struct AttnCfg {
+  static constexpr int kRowBytes = HD * 2 + 16;             // padded smem row (conflict-free ldmatrix)
+  static constexpr int kTileBytes = kKeyChunk * kRowBytes;  // one K or V chunk
+  static constexpr int kKV = 4 * kTileBytes;                // K and V, double-buffered
+  static constexpr int kQBytes = kMaxQV * kRowBytes;        // Q hi (or lo)
+  static constexpr int kQOff = kKV;
+  static constexpr int kPart = kMaxQV * (HD + 2) * 4;       // partial (o, m, l) per CTA
+  static constexpr int kPageOff = (kKV + 2 * kQBytes) > kPart ? (kKV + 2 * kQBytes) : kPart;
+  static constexpr int kSmem = kPageOff + kAttnPageCache * 4 + 256;
+};
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+// register-only (not volatile): the compiler may interleave independent MMAs
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2_trans(uint32_t& r0, uint32_t& r1, uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0,%1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr));
+}
+// two fp32 -> bf16x2 (lower-index element in the low half), plus the bf16 remainders
+__device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+  const __nv_bfloat16 l0 = __float2bfloat16_rn(x0 - __bfloat162float(h0));
+  const __nv_bfloat16 l1 = __float2bfloat16_rn(x1 - __bfloat162float(h1));
+  hi = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+  lo = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_size() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ float ld_dsmem(const float* local, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
+  return v;
+}
+
+// Page id of the page holding key position pos (-1: none or invalid, flagged).
+__device__ __forceinline__ int page_of(const AttnArgs& a, const int* pt, int pos) {
+  int page = -1;
+  if (pos / a.page_size < a.pt_ld) page = pt[pos / a.page_size];
+  if (page < 0 || page >= a.n_pages) {
+    set_status(a.status, ST_BAD_PAGE);
+    page = -1;
+  }
+  return page;
+}
+
+// K and V rows of one 64-key chunk into shared memory; positions past maxpos
+// (masked anyway) and bad pages become zeros.  spg: page ids of the pages
+// pg0, pg0 + 1, ... (nullptr: read the page table here).
+template <int HD>
+__device__ __forceinline__ void load_chunk(const AttnArgs& a, const int* pt, const int* spg, int pg0, int kvh,
+                                           int chunk, int maxpos, uint8_t* sK, uint8_t* sV, int tid) {
+  using C = AttnCfg<HD>;
+  constexpr int kCh = HD * 2 / 16;
+  for (int i = tid; i < kKeyChunk * kCh; i += kAttnThreads) {
+    const int key = i / kCh, ch = i % kCh;
+    const int pos = chunk * kKeyChunk + key;
+    uint8_t* dk = sK + key * C::kRowBytes + ch * 16;
+    uint8_t* dv = sV + key * C::kRowBytes + ch * 16;
+    int page = -1;
+    if (pos <= maxpos) page = spg ? spg[pos / a.page_size - pg0] : page_of(a, pt, pos);
+    if (page < 0) {
+      *reinterpret_cast<uint4*>(dk) = make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(dv) = make_uint4(0, 0, 0, 0);
+      continue;
+    }
+    const size_t off = (((size_t)page * a.hkv + kvh) * a.page_size + pos % a.page_size) * HD + ch * 8;
+    cp_async16(dk, a.kcache + off);
+    cp_async16(dv, a.vcache + off);
+  }
+  cp_async_commit();
+}
+
+// Partial attention of 4 warps (tid 0..127, warp = tid / 32) over key chunks
+// [c0, c1): rows row0..row0+nrows-1 of the row block (positions in s_pos),
+// query vectors qv = r * GROUP + head.  Leaves the unnormalised output and the
+// softmax (max, sum) of each query vector in smem as [64][HD + 2] floats.
+// bar() synchronises the 128 threads.  Each warp writes its own query vectors'
+// entries on return; the caller synchronises before reading other warps'.
+template <int HD, int GROUP, typename Bar>
+__device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0, int nrows, const int* s_pos,
+                             int maxpos, int c0, int c1, uint8_t* smem, int tid, Bar bar) {
+  using C = AttnCfg<HD>;
+  constexpr int KS = HD / 16;
+  constexpr int NT = HD / 8;
+  constexpr int NJ = kKeyChunk / 8;  // 8-key n-tiles per chunk
+  const int warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, c4 = lane & 3;
+  const int nqv = nrows * GROUP;
+  const int qa = warp * 16 + g, qb = qa + 8;
+  const int posa = qa < nqv ? s_pos[qa / GROUP] : -1, posb = qb < nqv ? s_pos[qb / GROUP] : -1;
+  uint8_t* sQh = smem + C::kQOff;
+  uint8_t* sQl = sQh + C::kQBytes;
+
+  // Q into shared memory as bf16 hi/lo rows (zeros past nqv); q is rewritten by
+  // every layer, by other CTAs of a persistent grid: L2 loads
+  constexpr int kQIter = kMaxQV * (HD / 4) / kAttnThreads;  // 8 or 16 float4 per thread
+  static_assert(kQIter % 4 == 0, "Q staging in groups of four");
+#pragma unroll 1
+  for (int i0 = 0; i0 < kQIter; i0 += 4) {
+    float4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = tid + (i0 + u) * kAttnThreads;
+      const int qv = i / (HD / 4), d4 = i % (HD / 4);
+      v[u] = qv < nqv ? __ldcg(reinterpret_cast<const float4*>(a.q + (size_t)(row0 + qv / GROUP) * a.q_ld +
+                                                               (kvh * GROUP + qv % GROUP) * HD) + d4)
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = tid + (i0 + u) * kAttnThreads;
+      const int qv = i / (HD / 4), d4 = i % (HD / 4);
+      uint2 h, l;
+      split2(v[u].x, v[u].y, h.x, l.x);
+      split2(v[u].z, v[u].w, h.y, l.y);
+      *reinterpret_cast<uint2*>(sQh + qv * C::kRowBytes + d4 * 8) = h;
+      *reinterpret_cast<uint2*>(sQl + qv * C::kRowBytes + d4 * 8) = l;
+    }
+  }
+
+  // page ids of the whole key range, one round of loads instead of one per key row
+  const int last = min(c1 * kKeyChunk - 1, maxpos);
+  const int pg0 = c0 * kKeyChunk / a.page_size;
+  const int npg = last >= c0 * kKeyChunk ? last / a.page_size + 1 - pg0 : 0;
+  int* spg = reinterpret_cast<int*>(smem + C::kPageOff);
+  const bool cached = npg <= kAttnPageCache;
+  if (cached)
+    for (int i = tid; i < npg; i += kAttnThreads) spg[i] = page_of(a, pt, (pg0 + i) * a.page_size);
+  bar();
+  const int* pgs = cached ? spg : nullptr;
+
+  float o[NT][4];
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
+  float ma = -INFINITY, mb = -INFINITY, la = 0.f, lb = 0.f;
+  const bool active = warp * 16 < nqv;
+  // ldmatrix.x4 row address of this lane in the warp's 16-row Q tile
+  const uint32_t qrow = (uint32_t)((warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * C::kRowBytes +
+                                   ((lane >> 4) & 1) * 16);
+  const uint32_t qh_base = smem_u32(sQh) + qrow, ql_base = smem_u32(sQl) + qrow;
+
+  if (c0 < c1) load_chunk<HD>(a, pt, pgs, pg0, kvh, c0, maxpos, smem, smem + C::kTileBytes, tid);
+  for (int ch = c0; ch < c1; ++ch) {
+    const int buf = (ch - c0) & 1;
+    const uint8_t* sK = smem + buf * 2 * C::kTileBytes;
+    const uint8_t* sV = sK + C::kTileBytes;
+    cp_async_wait_all();
+    bar();
+    if (ch + 1 < c1) {
+      uint8_t* nK = smem + (buf ^ 1) * 2 * C::kTileBytes;
+      load_chunk<HD>(a, pt, pgs, pg0, kvh, ch + 1, maxpos, nK, nK + C::kTileBytes, tid);
+    }
+    if (active) {
+      // S = Q K^T for the chunk's keys: NJ n-tiles of 8 keys, Q fragments per k-step
+      float s[NJ][4];
+#pragma unroll
+      for (int j = 0; j < NJ; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+#pragma unroll
+      for (int ks = 0; ks < KS; ++ks) {
+        uint32_t qh[4], ql[4], kb[NJ][2];
+        ldsm_x4(qh, qh_base + ks * 32);
+        ldsm_x4(ql, ql_base + ks * 32);
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) {
+          const uint8_t* krow = sK + (j * 8 + g) * C::kRowBytes;
+          kb[j][0] = *reinterpret_cast<const uint32_t*>(krow + (ks * 16 + 2 * c4) * 2);
+          kb[j][1] = *reinterpret_cast<const uint32_t*>(krow + (ks * 16 + 8 + 2 * c4) * 2);
+        }
+        // independent accumulators back to back; hi and lo products of one
+        // n-tile are NJ MMAs apart
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) mma_bf16_16816(s[j], qh, kb[j][0], kb[j][1]);
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) mma_bf16_16816(s[j], ql, kb[j][0], kb[j][1]);
+      }
+      // scale, causal mask, online softmax (rows qa and qb)
+      float mxa = -INFINITY, mxb = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < NJ; ++j) {
+        const int kp = ch * kKeyChunk + j * 8 + 2 * c4;
+        s[j][0] = kp <= posa ? s[j][0] * a.scale : -INFINITY;
+        s[j][1] = kp + 1 <= posa ? s[j][1] * a.scale : -INFINITY;
+        s[j][2] = kp <= posb ? s[j][2] * a.scale : -INFINITY;
+        s[j][3] = kp + 1 <= posb ? s[j][3] * a.scale : -INFINITY;
+        mxa = fmaxf(mxa, fmaxf(s[j][0], s[j][1]));
+        mxb = fmaxf(mxb, fmaxf(s[j][2], s[j][3]));
+      }
+      mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, 1));
+      mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, 2));
+      mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, 1));
+      mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, 2));
+      const float mna = fmaxf(ma, mxa), mnb = fmaxf(mb, mxb);
+      const float ca = mna == -INFINITY ? 1.f : expf(ma - mna);
+      const float cb = mnb == -INFINITY ? 1.f : expf(mb - mnb);
+      float sa = 0.f, sb = 0.f;
+#pragma unroll
+      for (int j = 0; j < NJ; ++j) {
+        s[j][0] = s[j][0] == -INFINITY ? 0.f : expf(s[j][0] - mna);
+        s[j][1] = s[j][1] == -INFINITY ? 0.f : expf(s[j][1] - mna);
+        s[j][2] = s[j][2] == -INFINITY ? 0.f : expf(s[j][2] - mnb);
+        s[j][3] = s[j][3] == -INFINITY ? 0.f : expf(s[j][3] - mnb);
+        sa += s[j][0] + s[j][1];
+        sb += s[j][2] + s[j][3];
+      }
+      sa += __shfl_xor_sync(0xffffffffu, sa, 1);
+      sa += __shfl_xor_sync(0xffffffffu, sa, 2);
+      sb += __shfl_xor_sync(0xffffffffu, sb, 1);
+      sb += __shfl_xor_sync(0xffffffffu, sb, 2);
+      la = la * ca + sa;
+      lb = lb * cb + sb;
+      ma = mna;
+      mb = mnb;
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        o[nt][0] *= ca; o[nt][1] *= ca; o[nt][2] *= cb; o[nt][3] *= cb;
+      }
+      // O += P V: P as A fragments (keys are the k dimension), V via ldmatrix.trans
+#pragma unroll
+      for (int kk = 0; kk < NJ / 2; ++kk) {
+        uint32_t ph[4], pl[4];
+        split2(s[2 * kk][0], s[2 * kk][1], ph[0], pl[0]);
+        split2(s[2 * kk][2], s[2 * kk][3], ph[1], pl[1]);
+        split2(s[2 * kk + 1][0], s[2 * kk + 1][1], ph[2], pl[2]);
+        split2(s[2 * kk + 1][2], s[2 * kk + 1][3], ph[3], pl[3]);
+        const uint32_t vrow = smem_u32(sV + (kk * 16 + (lane & 15)) * C::kRowBytes);
+#pragma unroll
+        for (int n0 = 0; n0 < NT; n0 += 4) {
+          uint32_t vb[4][2];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) ldsm_x2_trans(vb[u][0], vb[u][1], vrow + (n0 + u) * 16);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) mma_bf16_16816(o[n0 + u], ph, vb[u][0], vb[u][1]);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) mma_bf16_16816(o[n0 + u], pl, vb[u][0], vb[u][1]);
+        }
+      }
+    }
+  }
+  bar();  // K/V and Q buffers are reused for the partial results below
+
+  // partial (unnormalised o, m, l) of this CTA in its own shared memory
+  float* part = reinterpret_cast<float*>(smem);
+  if (active) {
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      const int d = nt * 8 + 2 * c4;
+      part[qa * (HD + 2) + d] = o[nt][0];
+      part[qa * (HD + 2) + d + 1] = o[nt][1];
+      part[qb * (HD + 2) + d] = o[nt][2];
+      part[qb * (HD + 2) + d + 1] = o[nt][3];
+    }
+    if (c4 == 0) {
+      part[qa * (HD + 2) + HD] = ma;
+      part[qa * (HD + 2) + HD + 1] = la;
+      part[qb * (HD + 2) + HD] = mb;
+      part[qb * (HD + 2) + HD + 1] = lb;
+    }
+  }
+}
+
+}  // namespace pard

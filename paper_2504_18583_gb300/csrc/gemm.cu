@@ -23,238 +23,9 @@
 //  * programmatic dependent launch: the weight tiles of the first stages
 //    are requested before waiting on the previous kernel, since weights do
 //    not depend on it.
-#include <climits>
-
-#include "common.cuh"
-#include "internal.h"
+#include "gemm_core.cuh"
 
 namespace pard {
-
-template <int TT>
-struct GemmCfg {
-  static constexpr int kABytes = kTileN * 128;       // 128 rows x 64 bf16
-  static constexpr int kBBytes = 2 * TT * 128;       // 2*TT rows x 64 bf16
-  static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStages = TT <= 16 ? 5 : (TT <= 32 ? 4 : 3);
-  static constexpr int kAccCols = 2 * TT;
-  static constexpr int kNumAcc = (2 * kAccCols <= 256) ? 2 : 1;
-  static constexpr int kTmemCols = kNumAcc * kAccCols <= 32 ? 32 : kNumAcc * kAccCols <= 64 ? 64
-                                   : kNumAcc * kAccCols <= 128 ? 128 : 256;
-  static constexpr int kChunks = TT / kEpiTok;
-  // scratch after the stage ring
-  static constexpr int kBarBytes = 8 * (2 * kStages + 4);
-  static constexpr int kMiscBytes = 64;
-  static constexpr int kScratchFloats = TT + 4 * 64 + 16 + kEpiTok * kTileN;
-  static constexpr int kSmem = 1024 + kStages * kStageBytes + kBarBytes + kMiscBytes + 4 * kScratchFloats;
-};
-
-__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
-
-__device__ __forceinline__ long owner_of(long u, long U, long G) { return ((u + 1) * G + U - 1) / U - 1; }
-__device__ __forceinline__ long range_start(long c, long U, long G) { return c * U / G; }
-
-__device__ __forceinline__ int seg_of(const GemmArgs& a, int w_tile) {
-  int s = 0;
-#pragma unroll
-  for (int i = 1; i < kMaxSeg; ++i)
-    if (i < a.nseg && w_tile >= a.seg_tile0[i]) s = i;
-  return s;
-}
-
-struct EpiSmem {
-  float* rs;     // [TT]   RMS row scale
-  float* red;    // [4][16]
-  int* redi;     // [4][16]
-  float* red2;   // [4][16]
-  int* redi2;    // [4][16]
-  float* tmx;    // [16]
-  float* xch;    // [16][128]
-};
-
-// One 16-token chunk of the epilogue for the thread holding weight row fr.
-__device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_tile, int tok0, int rs_off, int fr,
-                          int et, int M, const EpiSmem& S) {
-  const int q = fr >> 5, lane = fr & 31;
-  if (a.ssq_in) {
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) v[j] *= S.rs[rs_off + j];
-  }
-  if (a.mode == MODE_RESID) {
-    const int n = w_tile * kTileN + fr;
-    const bool nv = n < a.seg_rows[0];
-    const float g = nv ? __bfloat162float(a.g_next[n]) : 0.f;
-    float sq[kEpiTok];
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      const int m = tok0 + j;
-      float hn = 0.f;
-      if (m < M && nv) {
-        float* hp = a.h + (size_t)m * a.h_ld + n;
-        hn = *hp + v[j];
-        *hp = hn;
-        __nv_bfloat16 hi, lo;
-        split_bf16(hn * g, hi, lo);
-        a.x_next[xpk(2 * m, n, a.x_rows)] = hi;
-        a.x_next[xpk(2 * m + 1, n, a.x_rows)] = lo;
-      }
-      sq[j] = hn * hn;
-    }
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      const float s = warp_sum(sq[j]);
-      if (lane == 0) S.red[q * 16 + j] = s;
-    }
-    epi_bar();
-    if (et < kEpiTok) {
-      const int m = tok0 + et;
-      if (m < M)
-        a.ssq_out[(size_t)w_tile * a.m_cap + m] =
-            ((S.red[et] + S.red[16 + et]) + S.red[32 + et]) + S.red[48 + et];
-    }
-    epi_bar();
-  } else if (a.mode == MODE_QKV) {
-    const int seg = seg_of(a, w_tile);
-    const int n = (w_tile - a.seg_tile0[seg]) * kTileN + fr;
-    const bool nv = n < a.seg_rows[seg];
-    if (seg < 2) {
-#pragma unroll
-      for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
-      epi_bar();
-      const int half = a.hd >> 1, jj = n % a.hd;
-      const bool lo_half = jj < half;
-      const int pfr = lo_half ? fr + half : fr - half;
-      const int fi = lo_half ? jj : jj - half;
-#pragma unroll
-      for (int j = 0; j < kEpiTok; ++j) {
-        const int m = tok0 + j;
-        if (m < M) {
-          const int pos = a.row_pos[m];
-          const float2 cs = a.rope[(size_t)pos * half + fi];
-          const float p = S.xch[j * kTileN + pfr];
-          v[j] = lo_half ? v[j] * cs.x - p * cs.y : p * cs.y + v[j] * cs.x;
-        }
-      }
-      epi_bar();
-    }
-    if (nv) {
-#pragma unroll
-      for (int j = 0; j < kEpiTok; ++j) {
-        const int m = tok0 + j;
-        if (m >= M) continue;
-        if (seg == 0) {
-          a.q_out[(size_t)m * a.q_ld + n] = v[j];
-        } else {
-          const int pos = a.row_pos[m], b = a.row_seq[m];
-          if (pos < 0 || pos / a.page_size >= a.pt_ld) { set_status(a.status, ST_BAD_POS); continue; }
-          const int page = a.page_table[(size_t)b * a.pt_ld + pos / a.page_size];
-          if (page < 0 || page >= a.n_pages) { set_status(a.status, ST_BAD_PAGE); continue; }
-          const int kvh = n / a.hd, e = n % a.hd;
-          __nv_bfloat16* base = seg == 1 ? a.kcache : a.vcache;
-          base[(((size_t)page * a.hkv + kvh) * a.page_size + pos % a.page_size) * a.hd + e] =
-              __float2bfloat16_rn(v[j]);
-        }
-      }
-    }
-  } else if (a.mode == MODE_SWIGLU) {
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
-    epi_bar();
-    if (fr < 64) {
-      const int n = w_tile * 64 + fr;
-      if (n < a.seg_rows[0]) {
-#pragma unroll
-        for (int j = 0; j < kEpiTok; ++j) {
-          const int m = tok0 + j;
-          if (m >= M) continue;
-          const float gt = S.xch[j * kTileN + fr], up = S.xch[j * kTileN + 64 + fr];
-          __nv_bfloat16 hi, lo;
-          split_bf16(silu(gt) * up, hi, lo);
-          a.x_next[xpk(2 * m, n, a.x_rows)] = hi;
-          a.x_next[xpk(2 * m + 1, n, a.x_rows)] = lo;
-        }
-      }
-    }
-    epi_bar();
-  } else {  // MODE_LOGITS
-    const int vi = w_tile * kTileN + fr;
-    const bool valid = vi < a.vocab;
-    const float T = a.call->temp;
-    const bool sample = a.call->sample != 0 && a.row_gi != nullptr;
-    float x[kEpiTok];
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      const int m = tok0 + j;
-      x[j] = valid ? v[j] : -INFINITY;
-      if (a.logits && valid && m < M) {
-        const int orow = a.row_out ? a.row_out[m] : m;
-        if (orow >= 0) a.logits[(size_t)orow * a.vocab + vi] = v[j];
-      }
-    }
-    // tile max and argmax per row
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      float mv = x[j];
-      int mi = valid ? vi : INT_MAX;
-      warp_argmax(mv, mi);
-      if (lane == 0) { S.red[q * 16 + j] = mv; S.redi[q * 16 + j] = mi; }
-    }
-    // Gumbel-max draw per row (sampling draft rows only)
-    if (sample) {
-#pragma unroll 1
-      for (int j = 0; j < kEpiTok; ++j) {
-        const int m = tok0 + j;
-        float gv = -INFINITY;
-        int gi = INT_MAX;
-        if (m < M && valid) {
-          const int ri = a.row_gi[m];
-          if (ri >= 0) {
-            const uint32_t w = philox_word(a.call->seed, (uint32_t)a.gumbel_stream, a.call->step,
-                                           (uint32_t)a.row_seq[m], (uint32_t)ri, (uint32_t)vi);
-            gv = x[j] / T + gumbel(w);
-            gi = vi;
-          }
-        }
-        warp_argmax(gv, gi);
-        if (lane == 0) { S.red2[q * 16 + j] = gv; S.redi2[q * 16 + j] = gi; }
-      }
-    }
-    epi_bar();
-    if (et < kEpiTok) {
-      float mv = S.red[et];
-      int mi = S.redi[et];
-      for (int qq = 1; qq < 4; ++qq) argmax_merge(mv, mi, S.red[qq * 16 + et], S.redi[qq * 16 + et]);
-      S.tmx[et] = mv;
-      S.redi[et] = mi;  // keep the tile argmax
-      if (sample) {
-        float gv = S.red2[et];
-        int gi = S.redi2[et];
-        for (int qq = 1; qq < 4; ++qq) argmax_merge(gv, gi, S.red2[qq * 16 + et], S.redi2[qq * 16 + et]);
-        S.red2[et] = gv;
-        S.redi2[et] = gi;
-      }
-    }
-    epi_bar();
-    float e[kEpiTok];
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) e[j] = valid ? expf(x[j] / T - S.tmx[j] / T) : 0.f;
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      const float s = warp_sum(e[j]);
-      if (lane == 0) S.red[q * 16 + j] = s;
-    }
-    epi_bar();
-    if (et < kEpiTok) {
-      const int m = tok0 + et;
-      if (m < M) {
-        const float se = ((S.red[et] + S.red[16 + et]) + S.red[32 + et]) + S.red[48 + et];
-        const size_t o = (size_t)w_tile * a.m_cap + m;
-        a.stats[o] = make_float4(S.tmx[et], se, sample ? S.red2[et] : -INFINITY, 0.f);
-        a.stats_i[o] = make_int2(S.redi[et], sample ? S.redi2[et] : -1);
-      }
-    }
-    epi_bar();
-  }
-}
 
 template <int TT>
 __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ GemmArgs a) {
@@ -267,19 +38,13 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
   uint64_t* empty = full + C::kStages;
   uint64_t* accf = empty + C::kStages;
   uint64_t* acce = accf + 2;
-  uint32_t* misc = reinterpret_cast<uint32_t*>(acce + 2);
+  uint64_t* drain = acce + 2;
+  uint32_t* misc = reinterpret_cast<uint32_t*>(drain + 1);
   uint32_t* tmem_slot = misc;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
   int* bcast = reinterpret_cast<int*>(misc + 2);
   float* scratch = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(misc) + C::kMiscBytes);
-  EpiSmem S;
-  S.rs = scratch;
-  S.red = S.rs + TT;
-  S.redi = reinterpret_cast<int*>(S.red + 64);
-  S.red2 = reinterpret_cast<float*>(S.redi + 64);
-  S.redi2 = reinterpret_cast<int*>(S.red2 + 64);
-  S.tmx = reinterpret_cast<float*>(S.redi2 + 64);
-  S.xch = S.tmx + 16;
+  const EpiSmem S = carve_epi<TT>(scratch);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long U = (long)a.w_tiles * a.tok_tiles * a.kc;
@@ -290,6 +55,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     for (int b = 0; b < 2; ++b) { mbar_init(&accf[b], 1); mbar_init(&acce[b], 128); }
+    mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -298,6 +64,8 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  uint32_t armed[C::kStages];  // producer: times each ring slot was armed
+  for (int s = 0; s < C::kStages; ++s) armed[s] = 0;
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -366,6 +134,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       int pre_kk[C::kStages], pre_tok[C::kStages];
       for (int i = 0; i < npre; ++i) {
         mbar_arrive_expect_tx(&full[i], C::kStageBytes);
+        ++armed[i];
         issue_a(i);
         pre_kk[i] = kk;
         pre_tok[i] = tok_tile;
@@ -382,6 +151,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
           break;
         }
         mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+        ++armed[s];
         issue_a(s);
         issue_b(s, kk, tok_tile);
         advance();
@@ -443,25 +213,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       const int ab = seg_i % C::kNumAcc;
       const int w_tile = (int)(t / a.tok_tiles), tok_tile = (int)(t % a.tok_tiles);
       const int tok_base = tok_tile * TT;
-      if (a.ssq_in) {
-        // all partial sums of squares of this token tile in one round of loads,
-        // then a fixed-order sum per row (16 rows at a time through xch)
-        for (int c0 = 0; c0 < TT; c0 += kEpiTok) {
-          const int nld = a.ssq_tiles * kEpiTok;
-          for (int i = et; i < nld; i += 128) {
-            const int tile = i / kEpiTok, j = i % kEpiTok;
-            const int m = tok_base + c0 + j;
-            S.xch[i] = m < M ? __ldcg(a.ssq_in + (size_t)tile * a.m_cap + m) : 0.f;
-          }
-          epi_bar();
-          if (et < kEpiTok) {
-            float ss = 0.f;
-            for (int t2 = 0; t2 < a.ssq_tiles; ++t2) ss += S.xch[t2 * kEpiTok + et];
-            S.rs[c0 + et] = 1.0f / sqrtf(ss * a.inv_d + a.eps);
-          }
-          epi_bar();
-        }
-      }
+      if (a.ssq_in) epi_row_scale<TT>(a, tok_base, et, M, S);
       if (!mbar_wait(&accf[ab], (uint32_t)((seg_i / C::kNumAcc) & 1), abort_flag)) {
         if (et == 0) set_status(a.status, ST_TIMEOUT_EPI);
         *abort_flag = 1;
@@ -470,86 +222,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       tc_fence_after();
       epi_bar();
       const uint32_t tbase = tmem + ab * C::kAccCols + ((uint32_t)(q * 32) << 16);
-      const bool whole = (ub == t * a.kc) && (ue == (t + 1) * a.kc);
-      if (whole) {
-#pragma unroll 1
-        for (int ch = 0; ch < C::kChunks; ++ch) {
-          uint32_t r[32];
-          tmem_ld32(tbase + ch * 32, r);
-          float v[kEpiTok];
-#pragma unroll
-          for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
-          epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S);
-        }
-      } else {
-        const int slot = (ub == u0) ? 0 : 1;
-        float* mine = a.partials + ((size_t)c * 2 + slot) * (kTileN * TT);
-#pragma unroll 1
-        for (int ch = 0; ch < C::kChunks; ++ch) {
-          uint32_t r[32];
-          tmem_ld32(tbase + ch * 32, r);
-          float4* dst = reinterpret_cast<float4*>(mine + ((size_t)ch * kTileN + fr) * kEpiTok);
-#pragma unroll
-          for (int j4 = 0; j4 < 4; ++j4)
-            dst[j4] = make_float4(__uint_as_float(r[8 * j4 + 0]) + __uint_as_float(r[8 * j4 + 1]),
-                                  __uint_as_float(r[8 * j4 + 2]) + __uint_as_float(r[8 * j4 + 3]),
-                                  __uint_as_float(r[8 * j4 + 4]) + __uint_as_float(r[8 * j4 + 5]),
-                                  __uint_as_float(r[8 * j4 + 6]) + __uint_as_float(r[8 * j4 + 7]));
-        }
-        __threadfence();
-        epi_bar();
-        const long cf = owner_of(t * a.kc, U, G), cl = owner_of((t + 1) * a.kc - 1, U, G);
-        if (et == 0) {
-          const int old = atomicAdd(&a.counters[t], 1);
-          bcast[0] = (old == (int)(cl - cf)) ? 1 : 0;
-        }
-        epi_bar();
-        if (bcast[0]) {
-          __threadfence();
-#pragma unroll 1
-          for (int ch = 0; ch < C::kChunks; ++ch) {
-            uint32_t r[32];
-            tmem_ld32(tbase + ch * 32, r);
-            float v[kEpiTok];
-#pragma unroll
-            for (int j = 0; j < kEpiTok; ++j) v[j] = 0.f;
-            // contributors in CTA order, four partial tiles requested per round trip
-            for (long cc0 = cf; cc0 <= cl; cc0 += 4) {
-              float4 pv[4][4];
-#pragma unroll
-              for (int q4 = 0; q4 < 4; ++q4) {
-                const long cc = cc0 + q4;
-                if (cc <= cl && cc != c) {
-                  const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
-                  const float4* p = reinterpret_cast<const float4*>(
-                      a.partials + ((size_t)cc * 2 + sl) * (kTileN * TT) + ((size_t)ch * kTileN + fr) * kEpiTok);
-#pragma unroll
-                  for (int j4 = 0; j4 < 4; ++j4) pv[q4][j4] = __ldcg(p + j4);
-                }
-              }
-#pragma unroll
-              for (int q4 = 0; q4 < 4; ++q4) {
-                const long cc = cc0 + q4;
-                if (cc > cl) break;
-                if (cc == c) {
-#pragma unroll
-                  for (int j = 0; j < kEpiTok; ++j) v[j] += __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
-                } else {
-#pragma unroll
-                  for (int j4 = 0; j4 < 4; ++j4) {
-                    v[4 * j4 + 0] += pv[q4][j4].x;
-                    v[4 * j4 + 1] += pv[q4][j4].y;
-                    v[4 * j4 + 2] += pv[q4][j4].z;
-                    v[4 * j4 + 3] += pv[q4][j4].w;
-                  }
-                }
-              }
-            }
-            epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S);
-          }
-          if (et == 0) a.counters[t] = 0;
-        }
-      }
+      epi_segment<TT>(a, t, ub, ue, u0, U, G, c, tbase, w_tile, tok_base, fr, et, M, S, bcast);
       tc_fence_before();
       mbar_arrive(&acce[ab]);
       epi_bar();
@@ -559,6 +232,17 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
 
   tc_fence_before();
   __syncthreads();
+  if (*abort_flag) {
+    // let this CTA's copies and MMAs in flight land before its memory goes away
+    if (warp == 0 && lane == 0)
+      for (int s = 0; s < C::kStages; ++s)
+        if (armed[s]) mbar_drain(&full[s], (armed[s] - 1) & 1u);
+    if (warp == 1 && lane == 0) {
+      umma_commit(drain);
+      mbar_drain(drain, 0);
+    }
+    __syncthreads();
+  }
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();

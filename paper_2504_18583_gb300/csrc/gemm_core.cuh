@@ -1,0 +1,439 @@
+// Shared device code of the weight-streaming GEMM: tile configuration, the
+// fused epilogues and the split-K finish.  Included by the per-phase GEMM
+// kernel (gemm.cu) and the persistent decode kernel (fwd.cu).
+#pragma once
+
+#include <climits>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace pard {
+
+template <int TT>
+struct GemmCfg {
+  static constexpr int kABytes = kTileN * 128;       // 128 rows x 64 bf16
+  static constexpr int kBBytes = 2 * TT * 128;       // 2*TT rows x 64 bf16
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = TT <= 16 ? 5 : (TT <= 32 ? 4 : 3);
+  static constexpr int kAccCols = 2 * TT;
+  static constexpr int kNumAcc = (2 * kAccCols <= 256) ? 2 : 1;
+  static constexpr int kTmemCols = kNumAcc * kAccCols <= 32 ? 32 : kNumAcc * kAccCols <= 64 ? 64
+                                   : kNumAcc * kAccCols <= 128 ? 128 : 256;
+  static constexpr int kChunks = TT / kEpiTok;
+  // scratch after the stage ring
+  static constexpr int kBarBytes = 8 * (2 * kStages + 5);  // full, empty, accf x2, acce x2, drain
+  static constexpr int kMiscBytes = 64;
+  static constexpr int kScratchFloats = TT + 4 * 64 + 16 + kEpiTok * kTileN + 3 * kEpiTok;
+  static constexpr int kSmem = 1024 + kStages * kStageBytes + kBarBytes + kMiscBytes + 4 * kScratchFloats;
+};
+
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+// epi_bar that also returns whether any of the 128 threads passed v != 0, so
+// that all of them take the same branch after it
+__device__ __forceinline__ bool epi_bar_any(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, 1, 128, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)v)
+      : "memory");
+  return r != 0;
+}
+
+__device__ __forceinline__ long owner_of(long u, long U, long G) { return ((u + 1) * G + U - 1) / U - 1; }
+__device__ __forceinline__ long range_start(long c, long U, long G) { return c * U / G; }
+
+__device__ __forceinline__ int seg_of(const GemmArgs& a, int w_tile) {
+  int s = 0;
+#pragma unroll
+  for (int i = 1; i < kMaxSeg; ++i)
+    if (i < a.nseg && w_tile >= a.seg_tile0[i]) s = i;
+  return s;
+}
+
+struct EpiSmem {
+  float* rs;     // [TT]   RMS row scale
+  float* red;    // [4][16]
+  int* redi;     // [4][16]
+  float* red2;   // [4][16]
+  int* redi2;    // [4][16]
+  float* tmx;    // [16]
+  float* xch;    // [16][128]
+  int* ri;       // [3][16] per-row facts of the chunk, loaded once by 16 threads
+};
+
+// Carves the epilogue scratch (GemmCfg<TT>::kScratchFloats floats) at p.
+template <int TT>
+__device__ __forceinline__ EpiSmem carve_epi(float* p) {
+  EpiSmem S;
+  S.rs = p;
+  S.red = S.rs + TT;
+  S.redi = reinterpret_cast<int*>(S.red + 64);
+  S.red2 = reinterpret_cast<float*>(S.redi + 64);
+  S.redi2 = reinterpret_cast<int*>(S.red2 + 64);
+  S.tmx = reinterpret_cast<float*>(S.redi2 + 64);
+  S.xch = S.tmx + 16;
+  S.ri = reinterpret_cast<int*>(S.xch + kEpiTok * kTileN);
+  return S;
+}
+
+// Eight consecutive columns (col % 8 == 0) of activation row m as bf16 hi/lo
+// pairs in the packed layout: one 16-byte chunk in each of rows 2m and 2m+1.
+__device__ __forceinline__ void store_pair8(__nv_bfloat16* x, int m, int col, int x_rows, const float (&v)[8]) {
+  uint32_t h[4], l[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    __nv_bfloat16 h0, l0, h1, l1;
+    split_bf16(v[2 * e], h0, l0);
+    split_bf16(v[2 * e + 1], h1, l1);
+    h[e] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+    l[e] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+  }
+  *reinterpret_cast<uint4*>(x + xpk(2 * m, col, x_rows)) = make_uint4(h[0], h[1], h[2], h[3]);
+  *reinterpret_cast<uint4*>(x + xpk(2 * m + 1, col, x_rows)) = make_uint4(l[0], l[1], l[2], l[3]);
+}
+
+// One 16-token chunk of the epilogue for the thread holding weight row fr.
+static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_tile, int tok0, int rs_off, int fr,
+                          int et, int M, const EpiSmem& S) {
+  const int q = fr >> 5, lane = fr & 31;
+  if (a.ssq_in) {
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) v[j] *= S.rs[rs_off + j];
+  }
+  if (a.mode == MODE_RESID) {
+    const int n = w_tile * kTileN + fr;
+    const bool nv = n < a.seg_rows[0];
+    const float g = nv ? __bfloat162float(a.g_next[n]) : 0.f;
+    // every load of the residual first (one round trip), then the stores;
+    // L2 loads: other CTAs of a persistent grid update h
+    float hv[kEpiTok];
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) {
+      const int m = tok0 + j;
+      hv[j] = (m < M && nv) ? __ldcg(a.h + (size_t)m * a.h_ld + n) : 0.f;
+    }
+    float sq[kEpiTok];
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) {
+      const int m = tok0 + j;
+      float hn = 0.f;
+      if (m < M && nv) {
+        hn = hv[j] + v[j];
+        a.h[(size_t)m * a.h_ld + n] = hn;
+        __nv_bfloat16 hi, lo;
+        split_bf16(hn * g, hi, lo);
+        a.x_next[xpk(2 * m, n, a.x_rows)] = hi;
+        a.x_next[xpk(2 * m + 1, n, a.x_rows)] = lo;
+      }
+      sq[j] = hn * hn;
+    }
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) {
+      const float s = warp_sum(sq[j]);
+      if (lane == 0) S.red[q * 16 + j] = s;
+    }
+    epi_bar();
+    if (et < kEpiTok) {
+      const int m = tok0 + et;
+      if (m < M)
+        a.ssq_out[(size_t)w_tile * a.m_cap + m] =
+            ((S.red[et] + S.red[16 + et]) + S.red[32 + et]) + S.red[48 + et];
+    }
+    epi_bar();
+  } else if (a.mode == MODE_QKV) {
+    const int seg = seg_of(a, w_tile);
+    const int n = (w_tile - a.seg_tile0[seg]) * kTileN + fr;
+    const bool nv = n < a.seg_rows[seg];
+    // row facts of the chunk: position (-1: invalid) and KV page (-1: none)
+    if (et < kEpiTok) {
+      const int m = tok0 + et;
+      int pos = -1, page = -1;
+      if (m < M) {
+        pos = a.row_pos[m];
+        if (pos < 0 || pos / a.page_size >= a.pt_ld) {
+          set_status(a.status, ST_BAD_POS);
+          pos = -1;
+        } else if (seg > 0) {
+          page = a.page_table[(size_t)a.row_seq[m] * a.pt_ld + pos / a.page_size];
+          if (page < 0 || page >= a.n_pages) {
+            set_status(a.status, ST_BAD_PAGE);
+            page = -1;
+          }
+        }
+      }
+      S.ri[et] = pos;
+      S.ri[kEpiTok + et] = page;
+    }
+    epi_bar();
+    if (seg < 2) {
+#pragma unroll
+      for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
+      epi_bar();
+      const int half = a.hd >> 1, jj = n % a.hd;
+      const bool lo_half = jj < half;
+      const int pfr = lo_half ? fr + half : fr - half;
+      const int fi = lo_half ? jj : jj - half;
+#pragma unroll
+      for (int j = 0; j < kEpiTok; ++j) {
+        const int pos = S.ri[j];
+        if (pos >= 0) {
+          const float2 cs = a.rope[(size_t)pos * half + fi];
+          const float p = S.xch[j * kTileN + pfr];
+          v[j] = lo_half ? v[j] * cs.x - p * cs.y : p * cs.y + v[j] * cs.x;
+        }
+      }
+      epi_bar();
+    }
+    if (nv) {
+#pragma unroll
+      for (int j = 0; j < kEpiTok; ++j) {
+        const int m = tok0 + j;
+        if (m >= M) continue;
+        if (seg == 0) {
+          a.q_out[(size_t)m * a.q_ld + n] = v[j];
+        } else {
+          const int pos = S.ri[j], page = S.ri[kEpiTok + j];
+          if (page < 0) continue;
+          const int kvh = n / a.hd, e = n % a.hd;
+          __nv_bfloat16* base = seg == 1 ? a.kcache : a.vcache;
+          base[(((size_t)page * a.hkv + kvh) * a.page_size + pos % a.page_size) * a.hd + e] =
+              __float2bfloat16_rn(v[j]);
+        }
+      }
+    }
+    epi_bar();  // the row facts are rewritten by the next chunk
+  } else if (a.mode == MODE_SWIGLU) {
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
+    epi_bar();
+    // thread et: token et / 8, output columns 8 (et % 8) .. +8 of the tile's
+    // 64 (gate rows 0..63 and up rows 64..127 of the exchange); one 16-byte
+    // store per hi / lo row instead of 16 scalar ones
+    {
+      const int jl = et >> 3, c8 = (et & 7) * 8;
+      const int m = tok0 + jl, n0 = w_tile * 64 + c8;
+      if (m < M && n0 < a.seg_rows[0]) {
+        const float* gp = S.xch + jl * kTileN + c8;
+        float out[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) out[e] = silu(gp[e]) * gp[64 + e];
+        if (n0 + 8 <= a.seg_rows[0]) {
+          store_pair8(a.x_next, m, n0, a.x_rows, out);
+        } else {
+          for (int e = 0; e < 8 && n0 + e < a.seg_rows[0]; ++e) {
+            __nv_bfloat16 hi, lo;
+            split_bf16(out[e], hi, lo);
+            a.x_next[xpk(2 * m, n0 + e, a.x_rows)] = hi;
+            a.x_next[xpk(2 * m + 1, n0 + e, a.x_rows)] = lo;
+          }
+        }
+      }
+    }
+    epi_bar();
+  } else {  // MODE_LOGITS
+    const int vi = w_tile * kTileN + fr;
+    const bool valid = vi < a.vocab;
+    const float T = a.call->temp;
+    const bool sample = a.call->sample != 0 && a.row_gi != nullptr;
+    // row facts of the chunk: logits row (-1: none), Gumbel index (-1: none), sequence
+    if (et < kEpiTok) {
+      const int m = tok0 + et;
+      const bool in = m < M;
+      S.ri[et] = in ? (a.row_out ? a.row_out[m] : m) : -1;
+      S.ri[kEpiTok + et] = (in && sample) ? a.row_gi[m] : -1;
+      S.ri[2 * kEpiTok + et] = (in && sample) ? a.row_seq[m] : 0;
+    }
+    epi_bar();
+    float x[kEpiTok];
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) {
+      x[j] = valid ? v[j] : -INFINITY;
+      const int orow = S.ri[j];
+      if (a.logits && valid && orow >= 0) a.logits[(size_t)orow * a.vocab + vi] = v[j];
+    }
+    // tile max and argmax per row
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) {
+      float mv = x[j];
+      int mi = valid ? vi : INT_MAX;
+      warp_argmax(mv, mi);
+      if (lane == 0) { S.red[q * 16 + j] = mv; S.redi[q * 16 + j] = mi; }
+    }
+    // Gumbel-max draw per row (sampling draft rows only)
+    if (sample) {
+#pragma unroll 1
+      for (int j = 0; j < kEpiTok; ++j) {
+        const int m = tok0 + j;
+        float gv = -INFINITY;
+        int gi = INT_MAX;
+        if (m < M && valid) {
+          const int ri = S.ri[kEpiTok + j];
+          if (ri >= 0) {
+            const uint32_t w = philox_word(a.call->seed, (uint32_t)a.gumbel_stream, a.call->step,
+                                           (uint32_t)S.ri[2 * kEpiTok + j], (uint32_t)ri, (uint32_t)vi);
+            gv = x[j] / T + gumbel(w);
+            gi = vi;
+          }
+        }
+        warp_argmax(gv, gi);
+        if (lane == 0) { S.red2[q * 16 + j] = gv; S.redi2[q * 16 + j] = gi; }
+      }
+    }
+    epi_bar();
+    if (et < kEpiTok) {
+      float mv = S.red[et];
+      int mi = S.redi[et];
+      for (int qq = 1; qq < 4; ++qq) argmax_merge(mv, mi, S.red[qq * 16 + et], S.redi[qq * 16 + et]);
+      S.tmx[et] = mv;
+      S.redi[et] = mi;  // keep the tile argmax
+      if (sample) {
+        float gv = S.red2[et];
+        int gi = S.redi2[et];
+        for (int qq = 1; qq < 4; ++qq) argmax_merge(gv, gi, S.red2[qq * 16 + et], S.redi2[qq * 16 + et]);
+        S.red2[et] = gv;
+        S.redi2[et] = gi;
+      }
+    }
+    epi_bar();
+    float e[kEpiTok];
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) e[j] = valid ? expf(x[j] / T - S.tmx[j] / T) : 0.f;
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) {
+      const float s = warp_sum(e[j]);
+      if (lane == 0) S.red[q * 16 + j] = s;
+    }
+    epi_bar();
+    if (et < kEpiTok) {
+      const int m = tok0 + et;
+      if (m < M) {
+        const float se = ((S.red[et] + S.red[16 + et]) + S.red[32 + et]) + S.red[48 + et];
+        const size_t o = (size_t)w_tile * a.m_cap + m;
+        a.stats[o] = make_float4(S.tmx[et], se, sample ? S.red2[et] : -INFINITY, 0.f);
+        a.stats_i[o] = make_int2(S.redi[et], sample ? S.redi2[et] : -1);
+      }
+    }
+    epi_bar();
+  }
+}
+
+
+// Finish one segment [ub, ue) of tile t whose fp32 accumulator (hi/lo token
+// columns) sits at TMEM address tbase: the whole tile goes straight to the
+// epilogue; a partial tile writes its partial and the last CTA to arrive sums
+// all partials in CTA order and runs the epilogue.  Collective over the 128
+// epilogue threads.
+template <int TT>
+__device__ void epi_segment(const GemmArgs& a, long t, long ub, long ue, long u0, long U, long G, long c,
+                            uint32_t tbase, int w_tile, int tok_base, int fr, int et, int M, const EpiSmem& S,
+                            int* bcast) {
+  using C = GemmCfg<TT>;
+  const bool whole = (ub == t * a.kc) && (ue == (t + 1) * a.kc);
+  if (whole) {
+#pragma unroll 1
+    for (int ch = 0; ch < C::kChunks; ++ch) {
+      uint32_t r[32];
+      tmem_ld32(tbase + ch * 32, r);
+      float v[kEpiTok];
+#pragma unroll
+      for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
+      epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S);
+    }
+  } else {
+    const int slot = (ub == u0) ? 0 : 1;
+    float* mine = a.partials + ((size_t)c * 2 + slot) * (kTileN * TT);
+#pragma unroll 1
+    for (int ch = 0; ch < C::kChunks; ++ch) {
+      uint32_t r[32];
+      tmem_ld32(tbase + ch * 32, r);
+      float4* dst = reinterpret_cast<float4*>(mine + ((size_t)ch * kTileN + fr) * kEpiTok);
+#pragma unroll
+      for (int j4 = 0; j4 < 4; ++j4)
+        dst[j4] = make_float4(__uint_as_float(r[8 * j4 + 0]) + __uint_as_float(r[8 * j4 + 1]),
+                              __uint_as_float(r[8 * j4 + 2]) + __uint_as_float(r[8 * j4 + 3]),
+                              __uint_as_float(r[8 * j4 + 4]) + __uint_as_float(r[8 * j4 + 5]),
+                              __uint_as_float(r[8 * j4 + 6]) + __uint_as_float(r[8 * j4 + 7]));
+    }
+    // the barrier orders every thread's partial before the one acq_rel
+    // arrival (cumulative), which also acquires the earlier arrivals' partials
+    epi_bar();
+    const long cf = owner_of(t * a.kc, U, G), cl = owner_of((t + 1) * a.kc - 1, U, G);
+    if (et == 0) {
+      const int old = atom_add_acq_rel(&a.counters[t], 1);
+      bcast[0] = (old == (int)(cl - cf)) ? 1 : 0;
+    }
+    epi_bar();
+    if (bcast[0]) {
+#pragma unroll 1
+      for (int ch = 0; ch < C::kChunks; ++ch) {
+        uint32_t r[32];
+        tmem_ld32(tbase + ch * 32, r);
+        float v[kEpiTok];
+#pragma unroll
+        for (int j = 0; j < kEpiTok; ++j) v[j] = 0.f;
+        // contributors in CTA order, four partial tiles requested per round trip
+        for (long cc0 = cf; cc0 <= cl; cc0 += 4) {
+          float4 pv[4][4];
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4) {
+            const long cc = cc0 + q4;
+            if (cc <= cl && cc != c) {
+              const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
+              const float4* p = reinterpret_cast<const float4*>(
+                  a.partials + ((size_t)cc * 2 + sl) * (kTileN * TT) + ((size_t)ch * kTileN + fr) * kEpiTok);
+#pragma unroll
+              for (int j4 = 0; j4 < 4; ++j4) pv[q4][j4] = __ldcg(p + j4);
+            }
+          }
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4) {
+            const long cc = cc0 + q4;
+            if (cc > cl) break;
+            if (cc == c) {
+#pragma unroll
+              for (int j = 0; j < kEpiTok; ++j) v[j] += __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
+            } else {
+#pragma unroll
+              for (int j4 = 0; j4 < 4; ++j4) {
+                v[4 * j4 + 0] += pv[q4][j4].x;
+                v[4 * j4 + 1] += pv[q4][j4].y;
+                v[4 * j4 + 2] += pv[q4][j4].z;
+                v[4 * j4 + 3] += pv[q4][j4].w;
+              }
+            }
+          }
+        }
+        epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S);
+      }
+      if (et == 0) a.counters[t] = 0;
+    }
+  }
+}
+
+// RMS row scale for the token tile starting at tok_base: all partial sums of
+// squares in one round of loads, then a fixed-order sum per row.
+template <int TT>
+__device__ void epi_row_scale(const GemmArgs& a, int tok_base, int et, int M, const EpiSmem& S) {
+  for (int c0 = 0; c0 < TT; c0 += kEpiTok) {
+    const int nld = a.ssq_tiles * kEpiTok;
+    for (int i = et; i < nld; i += 128) {
+      const int tile = i / kEpiTok, j = i % kEpiTok;
+      const int m = tok_base + c0 + j;
+      S.xch[i] = m < M ? __ldcg(a.ssq_in + (size_t)tile * a.m_cap + m) : 0.f;
+    }
+    epi_bar();
+    if (et < kEpiTok) {
+      float ss = 0.f;
+      for (int t2 = 0; t2 < a.ssq_tiles; ++t2) ss += S.xch[t2 * kEpiTok + et];
+      S.rs[c0 + et] = 1.0f / sqrtf(ss * a.inv_d + a.eps);
+    }
+    epi_bar();
+  }
+}
+
+}  // namespace pard

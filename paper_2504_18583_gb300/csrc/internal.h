@@ -179,7 +179,37 @@ struct AcceptArgs {
   int* n_emit;
 };
 
-// launchers (gemm.cu, attention.cu, misc.cu)
+// Persistent decode pass: one launch runs every phase of every layer.
+enum PhaseType : int { PH_GEMM = 0, PH_ATTN = 1 };
+struct Phase {
+  int type;
+  int dep;            // phase whose completion this phase's inputs need (-1: none)
+  int attn_groups;    // PH_ATTN: (sequence, kv head, row block) groups
+  int attn_split;     // PH_ATTN: key splits per group
+  GemmArgs g;         // PH_GEMM (packed weights, one token tile)
+  AttnArgs at;        // PH_ATTN
+};
+struct FwdArgs {
+  const Phase* phases;   // device array
+  int n_phases;
+  unsigned* done;        // per-phase completion counters, monotonic over launches
+  unsigned target;       // a phase is complete when done[p] reaches target (launch count x grid)
+  float* attn_part;      // [groups * split][64][hd + 2] attention partials
+  int* attn_cnt;         // [groups] arrival counters (left at zero)
+  uint32_t* status;
+  const int* m_dev;
+  int m_cap;
+};
+constexpr int kFwdMaxAttnItems = 1024;  // (group, split) attention items of one persistent pass
+constexpr int kMaxQVRows = 64;          // query vectors of one attention work unit
+constexpr int kFwdTT = 16;              // persistent pass: token tile (rows of one pass, at most)
+constexpr int kFwdMaxSplit = 8;         // persistent pass: key splits per attention group
+constexpr int kFwdPrefetch = 8;         // persistent pass: weight units each CTA keeps requested into L2 ahead
+constexpr int kFwdPrefetchMax = 8;      // ... and at most this many while its ring waits on a phase
+
+// launchers (gemm.cu, attention.cu, misc.cu, fwd.cu)
+int fwd_smem_bytes(int hd);
+cudaError_t launch_fwd(const FwdArgs& f, int hd, int group, int grid, cudaStream_t s);
 void launch_embed(const EmbedArgs& a, int grid, cudaStream_t s, bool pdl);
 void launch_gather_rows(const __nv_bfloat16* x, int x_rows, const float* ssq, int ssq_tiles, int m_cap_src, int src_row,
                         __nv_bfloat16* xg, int xg_rows, float* ssqg, int m_cap_dst, int dst_row, int d, cudaStream_t s,

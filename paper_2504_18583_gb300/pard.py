@@ -76,6 +76,10 @@ def lib() -> ctypes.CDLL:
         L.pard_last_error.restype = ctypes.c_char_p
         L.pard_destroy.argtypes = [vp]
         L.pard_destroy.restype = None
+        L.pard_set_fused_pass.argtypes = [vp, i32]
+        L.pard_set_fused_pass.restype = ctypes.c_int
+        L.pard_fused_pass_used.argtypes = [vp]
+        L.pard_fused_pass_used.restype = i32
         for name in ("pard_load_weights", "pard_prefill", "pard_draft", "pard_verify", "pard_accept_commit",
                      "pard_set_logits", "pard_get_state", "pard_read_kv", "pard_last_status"):
             getattr(L, name).restype = ctypes.c_int
@@ -260,3 +264,11 @@ class PardEngine:
 
     def launch_count(self) -> int:
         return lib().pard_launch_count(self.ctx)
+
+    def set_fused_pass(self, enable: bool) -> None:
+        """Persistent single-kernel forward for small passes (default off); applies from the next prefill."""
+        _check(lib().pard_set_fused_pass(self.ctx, 1 if enable else 0), "pard_set_fused_pass")
+
+    def fused_pass_used(self) -> bool:
+        """True when the last draft / verify ran as one persistent kernel."""
+        return bool(lib().pard_fused_pass_used(self.ctx))

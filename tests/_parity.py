@@ -29,7 +29,7 @@ def margin(row: np.ndarray) -> float:
 class Pair:
     """GPU engine and oracle decoder on identical weights and page orders."""
 
-    def __init__(self, wl, draft_is_target: bool = False, prefill_chunk: int = 64):
+    def __init__(self, wl, draft_is_target: bool = False, prefill_chunk: int = 64, fused: bool = True):
         import torch
         from paper_2504_18583_gb300 import pard
         self.wl = wl
@@ -49,6 +49,7 @@ class Pair:
         self.eng = pard.PardEngine(wl.target, self.tw_dev, dshape, self.dw_dev, max_batch=wl.batch, max_k=wl.K,
                                    max_ctx=max_ctx, n_pages=n_pages, prefill_chunk=prefill_chunk,
                                    page_order_target=self.order_t, page_order_draft=self.order_d)
+        self.eng.set_fused_pass(fused)
         self.torch = torch
         self.stats = dict(excused_tokens=0, checked_tokens=0, max_logit_err=0.0, max_draft_logit_err=0.0)
 

@@ -33,10 +33,17 @@ def run_greedy(P: Pair, max_steps=64, inject_fn=None):
     return outs
 
 
-def test_tiny_greedy_matches_oracle_every_step():
+@pytest.mark.parametrize("fused", [True, False], ids=["persistent", "per_phase"])
+def test_tiny_greedy_matches_oracle_every_step(fused):
+    """Both forward-pass paths: the persistent kernel (draft 8 rows, verify 5
+    rows; FFN 768 so every matrix takes the packed layout it needs) and one
+    kernel per phase (FFN 688: ragged row-major gate/up/down)."""
     wl = S.WORKLOADS["tiny"]
-    P = Pair(wl)
+    if fused:
+        wl = wl.replace(target=wl.target.replace(ffn=768), draft=wl.draft.replace(ffn=768))
+    P = Pair(wl, fused=fused)
     run_greedy(P)
+    assert P.eng.fused_pass_used() == fused
     assert P.oracle.all_done()
     # the generated sequence equals autoregressive greedy decoding where margins are clear
     assert P.stats["excused_tokens"] <= P.stats["checked_tokens"] // 10
@@ -48,8 +55,11 @@ def test_tiny_greedy_jittered_norms_batch_ragged():
     several offsets), norm gains != 1, prefill chunks of 64 rows."""
     wl = S.WORKLOADS["tiny"].replace(batch=3, prompt_len=None, prompt_len_range=(17, 50), norm_jitter=0.1,
                                      n_new=20)
+    wl = wl.replace(target=wl.target.replace(ffn=768), draft=wl.draft.replace(ffn=768))
     P = Pair(wl)
     run_greedy(P)
+    # 3 x 8 draft rows exceed one persistent pass; the 3 x 5 verify rows fit
+    assert P.eng.fused_pass_used()
     print("stats", P.stats)
 
 
@@ -109,16 +119,18 @@ def test_kv_cache_holds_the_oracle_keys_and_values():
             assert np.abs(v - vo).max() <= 0.02 * max(1.0, np.abs(vo).max())
 
 
-def test_full_width_8b_layers_short_prompt():
+@pytest.mark.parametrize("fused", [True, False], ids=["persistent", "per_phase"])
+def test_full_width_8b_layers_short_prompt(fused):
     """8B-shaped target and 1B-shaped draft at full width (every GEMM,
     attention and LM-head tile count of the full models), two layers each,
-    64-token prompt, three steps."""
+    64-token prompt, three steps; K = 8 gives 16 draft rows and 9 verify rows."""
     wl = S.WORKLOADS["8b_greedy"].replace(target=S.TARGET_8B.replace(n_layers=2),
                                           draft=S.DRAFT_1B.replace(n_layers=2), prompt_len=64, n_new=20)
-    P = Pair(wl, prefill_chunk=64)
+    P = Pair(wl, prefill_chunk=64, fused=fused)
     P.prefill()
     for step in range(1, 4):
         greedy_step(P, step)
+    assert P.eng.fused_pass_used() == fused
     assert P.eng.last_status() == 0
     print("stats", P.stats)
 
