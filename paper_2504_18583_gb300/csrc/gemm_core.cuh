@@ -105,50 +105,69 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
 #pragma unroll
     for (int j = 0; j < kEpiTok; ++j) v[j] *= S.rs[rs_off + j];
   }
+  // Row-major phase: after the accumulator columns are exchanged through
+  // S.xch, thread et handles token jl = et / 8 and the 16 consecutive tile rows
+  // (output columns) c16 .. c16+15, c16 = 16 (et % 8), so the stores are
+  // 16-byte vectors instead of one scalar per token.
+  const int jl = et >> 3, c16 = (et & 7) * 16;
+  const int mr = tok0 + jl;  // this thread's token in the row-major phase
   if (a.mode == MODE_RESID) {
-    const int n = w_tile * kTileN + fr;
-    const bool nv = n < a.seg_rows[0];
-    const float g = nv ? __bfloat162float(a.g_next[n]) : 0.f;
-    // every load of the residual first (one round trip), then the stores;
-    // L2 loads: other CTAs of a persistent grid update h
-    float hv[kEpiTok];
 #pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      const int m = tok0 + j;
-      hv[j] = (m < M && nv) ? __ldcg(a.h + (size_t)m * a.h_ld + n) : 0.f;
-    }
-    float sq[kEpiTok];
+    for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
+    epi_bar();
+    const int n0 = w_tile * kTileN + c16;
+    float sq = 0.f;
+    if (mr < M && n0 < a.seg_rows[0]) {
+      const float* xv = S.xch + jl * kTileN + c16;
+      float* hp = a.h + (size_t)mr * a.h_ld + n0;
+      if (n0 + 16 <= a.seg_rows[0] && (reinterpret_cast<uintptr_t>(a.g_next) & 15) == 0) {
+        // every load first (one round trip; L2: other CTAs of a persistent
+        // grid update h), then the stores
+        float4 hv[4];
+        uint4 gv[2];
 #pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      const int m = tok0 + j;
-      float hn = 0.f;
-      if (m < M && nv) {
-        hn = hv[j] + v[j];
-        a.h[(size_t)m * a.h_ld + n] = hn;
-        __nv_bfloat16 hi, lo;
-        split_bf16(hn * g, hi, lo);
-        a.x_next[xpk(2 * m, n, a.x_rows)] = hi;
-        a.x_next[xpk(2 * m + 1, n, a.x_rows)] = lo;
+        for (int i = 0; i < 4; ++i) hv[i] = __ldcg(reinterpret_cast<const float4*>(hp) + i);
+#pragma unroll
+        for (int i = 0; i < 2; ++i) gv[i] = *reinterpret_cast<const uint4*>(a.g_next + n0 + 8 * i);
+        float hn[16];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          hn[4 * i + 0] = hv[i].x + xv[4 * i + 0];
+          hn[4 * i + 1] = hv[i].y + xv[4 * i + 1];
+          hn[4 * i + 2] = hv[i].z + xv[4 * i + 2];
+          hn[4 * i + 3] = hv[i].w + xv[4 * i + 3];
+          reinterpret_cast<float4*>(hp)[i] = make_float4(hn[4 * i], hn[4 * i + 1], hn[4 * i + 2], hn[4 * i + 3]);
+        }
+        const __nv_bfloat16* gb = reinterpret_cast<const __nv_bfloat16*>(gv);
+#pragma unroll
+        for (int h8 = 0; h8 < 2; ++h8) {
+          float o[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) o[e] = hn[8 * h8 + e] * __bfloat162float(gb[8 * h8 + e]);
+          store_pair8(a.x_next, mr, n0 + 8 * h8, a.x_rows, o);
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) sq += hn[i] * hn[i];
+      } else {
+        for (int i = 0; i < 16 && n0 + i < a.seg_rows[0]; ++i) {
+          const float hn = __ldcg(hp + i) + xv[i];
+          hp[i] = hn;
+          __nv_bfloat16 hi, lo;
+          split_bf16(hn * __bfloat162float(a.g_next[n0 + i]), hi, lo);
+          a.x_next[xpk(2 * mr, n0 + i, a.x_rows)] = hi;
+          a.x_next[xpk(2 * mr + 1, n0 + i, a.x_rows)] = lo;
+          sq += hn * hn;
+        }
       }
-      sq[j] = hn * hn;
     }
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      const float s = warp_sum(sq[j]);
-      if (lane == 0) S.red[q * 16 + j] = s;
-    }
-    epi_bar();
-    if (et < kEpiTok) {
-      const int m = tok0 + et;
-      if (m < M)
-        a.ssq_out[(size_t)w_tile * a.m_cap + m] =
-            ((S.red[et] + S.red[16 + et]) + S.red[32 + et]) + S.red[48 + et];
-    }
-    epi_bar();
+    // the tile's sum of squares of this token: its 8 threads are 8 adjacent lanes
+    sq += __shfl_xor_sync(0xffffffffu, sq, 1);
+    sq += __shfl_xor_sync(0xffffffffu, sq, 2);
+    sq += __shfl_xor_sync(0xffffffffu, sq, 4);
+    if ((et & 7) == 0 && mr < M) a.ssq_out[(size_t)w_tile * a.m_cap + mr] = sq;
+    epi_bar();  // S.xch is rewritten by the next chunk
   } else if (a.mode == MODE_QKV) {
     const int seg = seg_of(a, w_tile);
-    const int n = (w_tile - a.seg_tile0[seg]) * kTileN + fr;
-    const bool nv = n < a.seg_rows[seg];
     // row facts of the chunk: position (-1: invalid) and KV page (-1: none)
     if (et < kEpiTok) {
       const int m = tok0 + et;
@@ -169,44 +188,57 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
       S.ri[et] = pos;
       S.ri[kEpiTok + et] = page;
     }
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
     epi_bar();
-    if (seg < 2) {
+    const int n0 = (w_tile - a.seg_tile0[seg]) * kTileN + c16;  // first column within the segment
+    const int pos = S.ri[jl];
+    if (mr < M && n0 < a.seg_rows[seg] && pos >= 0) {
+      const float* xv = S.xch + jl * kTileN;
+      float o[16];
 #pragma unroll
-      for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
-      epi_bar();
-      const int half = a.hd >> 1, jj = n % a.hd;
-      const bool lo_half = jj < half;
-      const int pfr = lo_half ? fr + half : fr - half;
-      const int fi = lo_half ? jj : jj - half;
+      for (int i = 0; i < 16; ++i) o[i] = xv[c16 + i];
+      if (seg < 2) {
+        // rotate-half RoPE: the 16 columns lie in one half of one head, and the
+        // partner half of that head is in the same 128-row tile
+        const int half = a.hd >> 1, jj = n0 % a.hd;
+        const bool lo_half = jj < half;
+        const int fi0 = lo_half ? jj : jj - half;
+        const int pc = lo_half ? c16 + half : c16 - half;
+        const float4* csp = reinterpret_cast<const float4*>(a.rope + (size_t)pos * half + fi0);
+        float4 cs4[8];
 #pragma unroll
-      for (int j = 0; j < kEpiTok; ++j) {
-        const int pos = S.ri[j];
-        if (pos >= 0) {
-          const float2 cs = a.rope[(size_t)pos * half + fi];
-          const float p = S.xch[j * kTileN + pfr];
-          v[j] = lo_half ? v[j] * cs.x - p * cs.y : p * cs.y + v[j] * cs.x;
+        for (int i = 0; i < 8; ++i) cs4[i] = csp[i];  // 16 (cos, sin) pairs
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float c = (i & 1) ? cs4[i >> 1].z : cs4[i >> 1].x;
+          const float sn = (i & 1) ? cs4[i >> 1].w : cs4[i >> 1].y;
+          const float p = xv[pc + i];
+          o[i] = lo_half ? o[i] * c - p * sn : p * sn + o[i] * c;
         }
       }
-      epi_bar();
-    }
-    if (nv) {
+      if (seg == 0) {
+        float4* qp = reinterpret_cast<float4*>(a.q_out + (size_t)mr * a.q_ld + n0);
 #pragma unroll
-      for (int j = 0; j < kEpiTok; ++j) {
-        const int m = tok0 + j;
-        if (m >= M) continue;
-        if (seg == 0) {
-          a.q_out[(size_t)m * a.q_ld + n] = v[j];
-        } else {
-          const int pos = S.ri[j], page = S.ri[kEpiTok + j];
-          if (page < 0) continue;
-          const int kvh = n / a.hd, e = n % a.hd;
+        for (int i = 0; i < 4; ++i) qp[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+      } else {
+        const int page = S.ri[kEpiTok + jl];
+        if (page >= 0) {
+          const int kvh = n0 / a.hd, e0 = n0 % a.hd;
           __nv_bfloat16* base = seg == 1 ? a.kcache : a.vcache;
-          base[(((size_t)page * a.hkv + kvh) * a.page_size + pos % a.page_size) * a.hd + e] =
-              __float2bfloat16_rn(v[j]);
+          __nv_bfloat16* dst =
+              base + (((size_t)page * a.hkv + kvh) * a.page_size + pos % a.page_size) * a.hd + e0;
+          uint32_t w[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            w[i] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(o[2 * i])) |
+                   ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(o[2 * i + 1])) << 16);
+          reinterpret_cast<uint4*>(dst)[0] = make_uint4(w[0], w[1], w[2], w[3]);
+          reinterpret_cast<uint4*>(dst)[1] = make_uint4(w[4], w[5], w[6], w[7]);
         }
       }
     }
-    epi_bar();  // the row facts are rewritten by the next chunk
+    epi_bar();  // S.xch and the row facts are rewritten by the next chunk
   } else if (a.mode == MODE_SWIGLU) {
 #pragma unroll
     for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
