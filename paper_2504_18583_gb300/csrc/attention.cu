@@ -8,11 +8,11 @@
 // Work unit: one sequence, one KV head, a block of rows times the query
 // heads that share the KV head (<= 64 query vectors, 16 per warp), and one
 // share of the key range.  The key range is split over the CTAs of one
-// thread-block cluster (<= 8); each CTA walks its 64-key chunks with K/V
+// thread-block cluster (<= 8); each CTA walks its 32-key chunks with K/V
 // pages double-buffered in shared memory (cp.async), computes S = Q K^T and
-// O += P V on the tensor cores (mma.sync m16n8k16, bf16 inputs, fp32
-// accumulators; Q and P carried as bf16 hi/lo pairs so the products keep
-// fp32-level accuracy against the bf16 cache), and keeps the online-softmax
+// O += P V on the tensor cores (mma.sync m16n8k16, fp16 inputs, fp32
+// accumulators: Q and P rounded to fp16, the bf16 K/V converted to fp16 in
+// shared memory, which is exact in fp16's range), and keeps the online-softmax
 // state in registers.  The cluster then combines its partial (max, sum, O)
 // through distributed shared memory, in rank order, and writes the output
 // as bf16 hi/lo pairs in the packed activation layout of the O projection.
@@ -56,33 +56,51 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
   float* part = reinterpret_cast<float*>(smem);
   cluster_sync();
   // combine in rank order; CTA `rank` finishes query vectors rank, rank+NS, ...
+  // Every rank's value is requested before any is used (the loads overlap).
   for (int qv = (int)rank + (int)NS * (int)threadIdx.x; qv < nqv; qv += (int)NS * kAttnThreads) {
+    float2 ml[kMaxCluster];
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r)
+      ml[r] = r < (int)NS ? ld_dsmem2(part + qv * (HD + 2) + HD, (uint32_t)r) : make_float2(-INFINITY, 0.f);
     float mx = -INFINITY;
-    for (uint32_t r = 0; r < NS; ++r) mx = fmaxf(mx, ld_dsmem(part + qv * (HD + 2) + HD, r));
-    float L = 0.f;
-    for (uint32_t r = 0; r < NS; ++r) {
-      const float mr = ld_dsmem(part + qv * (HD + 2) + HD, r);
-      const float w = mr == -INFINITY ? 0.f : expf(mr - mx);
-      s_w[qv][r] = w;
-      L += ld_dsmem(part + qv * (HD + 2) + HD + 1, r) * w;
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r) mx = fmaxf(mx, ml[r].x);
+    float w[kMaxCluster], L = 0.f;
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r) {
+      w[r] = ml[r].x == -INFINITY ? 0.f : expf(ml[r].x - mx);
+      L += ml[r].y * w[r];
     }
-    for (uint32_t r = 0; r < NS; ++r) s_w[qv][r] /= L;
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r)
+      if (r < (int)NS) s_w[qv][r] = w[r] / L;
   }
   __syncthreads();
   const int my_qv = nqv > (int)rank ? (nqv - (int)rank + (int)NS - 1) / (int)NS : 0;
-  for (int i = threadIdx.x; i < my_qv * HD; i += kAttnThreads) {
-    const int qv = (int)rank + (int)NS * (i / HD), d = i % HD;
-    float acc = 0.f;
-    for (uint32_t r = 0; r < NS; ++r) {
-      const float w = s_w[qv][r];
-      if (w != 0.f) acc += ld_dsmem(part + qv * (HD + 2) + d, r) * w;
+  for (int i = threadIdx.x; i < my_qv * (HD / 2); i += kAttnThreads) {
+    const int qv = (int)rank + (int)NS * (i / (HD / 2)), d = 2 * (i % (HD / 2));
+    float2 pv[kMaxCluster];
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r)
+      pv[r] = r < (int)NS ? ld_dsmem2(part + qv * (HD + 2) + d, (uint32_t)r) : make_float2(0.f, 0.f);
+    float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r) {
+      const float wr = r < (int)NS ? s_w[qv][r] : 0.f;
+      if (wr != 0.f) {
+        acc.x += pv[r].x * wr;
+        acc.y += pv[r].y * wr;
+      }
     }
     const int m = row0 + qv / GROUP;
     const int col = (kvh * GROUP + qv % GROUP) * HD + d;
-    __nv_bfloat16 hi, lo;
-    split_bf16(acc, hi, lo);
-    a.x_out[xpk(2 * m, col, a.x_rows)] = hi;
-    a.x_out[xpk(2 * m + 1, col, a.x_rows)] = lo;
+    __nv_bfloat16 h0, l0, h1, l1;
+    split_bf16(acc.x, h0, l0);
+    split_bf16(acc.y, h1, l1);
+    *reinterpret_cast<uint32_t*>(a.x_out + xpk(2 * m, col, a.x_rows)) =
+        (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+    *reinterpret_cast<uint32_t*>(a.x_out + xpk(2 * m + 1, col, a.x_rows)) =
+        (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
   }
   cluster_sync();  // peers may still be reading this CTA's partial
 }

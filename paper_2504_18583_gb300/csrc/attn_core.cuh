@@ -4,6 +4,8 @@
 // and the persistent decode kernel (fwd_kernel.cuh).
 #pragma once
 
+#include <cuda_fp16.h>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -15,18 +17,18 @@ constexpr int kKeyChunk = 32;
 constexpr int kMaxCluster = 8;
 constexpr int kAttnPageCache = 512;  // page ids of one work unit's key range held in shared memory
 
-// Shared memory of one work unit: K and V chunks double-buffered, Q as bf16
-// hi and lo rows (the MMA A operand, read with ldmatrix), then the page id
-// cache; the partial result (o, m, l) reuses the front at the end.
+// Shared memory of one work unit: K and V chunks double-buffered, Q as fp16
+// rows (the MMA A operand, read with ldmatrix), then the page id cache; the
+// partial result (o, m, l) reuses the front at the end.
 template <int HD>
 struct AttnCfg {
   static constexpr int kRowBytes = HD * 2 + 16;             // padded smem row (conflict-free ldmatrix)
   static constexpr int kTileBytes = kKeyChunk * kRowBytes;  // one K or V chunk
   static constexpr int kKV = 4 * kTileBytes;                // K and V, double-buffered
-  static constexpr int kQBytes = kMaxQV * kRowBytes;        // Q hi (or lo)
+  static constexpr int kQBytes = kMaxQV * kRowBytes;        // Q rows
   static constexpr int kQOff = kKV;
   static constexpr int kPart = kMaxQV * (HD + 2) * 4;       // partial (o, m, l) per CTA
-  static constexpr int kPageOff = (kKV + 2 * kQBytes) > kPart ? (kKV + 2 * kQBytes) : kPart;
+  static constexpr int kPageOff = (kKV + kQBytes) > kPart ? (kKV + kQBytes) : kPart;
   static constexpr int kSmem = kPageOff + kAttnPageCache * 4 + 256;
 };
 
@@ -37,12 +39,21 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 // register-only (not volatile): the compiler may interleave independent MMAs
-__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-  asm(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// two fp32 -> fp16x2 (lower-index element in the low half)
+__device__ __forceinline__ uint32_t pack_h2(float x0, float x1) {
+  const __half2 h = __floats2half2_rn(x0, x1);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+// bf16x2 -> fp16x2; exact for magnitudes in [2^-14, 65504] (fp16 keeps more
+// significand bits than bf16), rounded below, infinite above
+__device__ __forceinline__ uint32_t bf2_to_h2(uint32_t x) {
+  return pack_h2(__uint_as_float(x << 16), __uint_as_float(x & 0xffff0000u));
 }
 __device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
@@ -51,14 +62,6 @@ __device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
 }
 __device__ __forceinline__ void ldsm_x2_trans(uint32_t& r0, uint32_t& r1, uint32_t addr) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0,%1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr));
-}
-// two fp32 -> bf16x2 (lower-index element in the low half), plus the bf16 remainders
-__device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
-  const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
-  const __nv_bfloat16 l0 = __float2bfloat16_rn(x0 - __bfloat162float(h0));
-  const __nv_bfloat16 l1 = __float2bfloat16_rn(x1 - __bfloat162float(h1));
-  hi = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-  lo = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
 }
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
@@ -73,11 +76,12 @@ __device__ __forceinline__ uint32_t cluster_size() {
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-__device__ __forceinline__ float ld_dsmem(const float* local, uint32_t rank) {
+// two consecutive floats (8-byte aligned) of CTA `rank`'s shared memory
+__device__ __forceinline__ float2 ld_dsmem2(const float* local, uint32_t rank) {
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
+  float2 v;
+  asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(remote) : "memory");
   return v;
 }
 
@@ -119,6 +123,22 @@ __device__ __forceinline__ void load_chunk(const AttnArgs& a, const int* pt, con
   cp_async_commit();
 }
 
+// The same thread's pieces of a landed chunk (load_chunk's mapping), bf16 ->
+// fp16 in place; zero-filled pieces are zeros in both formats.
+template <int HD>
+__device__ __forceinline__ void chunk_to_f16(uint8_t* sK, uint8_t* sV, int tid) {
+  using C = AttnCfg<HD>;
+  constexpr int kCh = HD * 2 / 16;
+  for (int i = tid; i < kKeyChunk * kCh; i += kAttnThreads) {
+    const int key = i / kCh, ch = i % kCh;
+    uint4* pk = reinterpret_cast<uint4*>(sK + key * C::kRowBytes + ch * 16);
+    uint4* pv = reinterpret_cast<uint4*>(sV + key * C::kRowBytes + ch * 16);
+    const uint4 k = *pk, v = *pv;
+    *pk = make_uint4(bf2_to_h2(k.x), bf2_to_h2(k.y), bf2_to_h2(k.z), bf2_to_h2(k.w));
+    *pv = make_uint4(bf2_to_h2(v.x), bf2_to_h2(v.y), bf2_to_h2(v.z), bf2_to_h2(v.w));
+  }
+}
+
 // Partial attention of 4 warps (tid 0..127, warp = tid / 32) over key chunks
 // [c0, c1): rows row0..row0+nrows-1 of the row block (positions in s_pos),
 // query vectors qv = r * GROUP + head.  Leaves the unnormalised output and the
@@ -137,11 +157,10 @@ __device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0
   const int nqv = nrows * GROUP;
   const int qa = warp * 16 + g, qb = qa + 8;
   const int posa = qa < nqv ? s_pos[qa / GROUP] : -1, posb = qb < nqv ? s_pos[qb / GROUP] : -1;
-  uint8_t* sQh = smem + C::kQOff;
-  uint8_t* sQl = sQh + C::kQBytes;
+  uint8_t* sQ = smem + C::kQOff;
 
-  // Q into shared memory as bf16 hi/lo rows (zeros past nqv); q is rewritten by
-  // every layer, by other CTAs of a persistent grid: L2 loads
+  // Q into shared memory as fp16 rows (zeros past nqv); q is rewritten by every
+  // layer, by other CTAs of a persistent grid: L2 loads
   constexpr int kQIter = kMaxQV * (HD / 4) / kAttnThreads;  // 8 or 16 float4 per thread
   static_assert(kQIter % 4 == 0, "Q staging in groups of four");
 #pragma unroll 1
@@ -159,11 +178,8 @@ __device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0
     for (int u = 0; u < 4; ++u) {
       const int i = tid + (i0 + u) * kAttnThreads;
       const int qv = i / (HD / 4), d4 = i % (HD / 4);
-      uint2 h, l;
-      split2(v[u].x, v[u].y, h.x, l.x);
-      split2(v[u].z, v[u].w, h.y, l.y);
-      *reinterpret_cast<uint2*>(sQh + qv * C::kRowBytes + d4 * 8) = h;
-      *reinterpret_cast<uint2*>(sQl + qv * C::kRowBytes + d4 * 8) = l;
+      *reinterpret_cast<uint2*>(sQ + qv * C::kRowBytes + d4 * 8) =
+          make_uint2(pack_h2(v[u].x, v[u].y), pack_h2(v[u].z, v[u].w));
     }
   }
 
@@ -186,14 +202,15 @@ __device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0
   // ldmatrix.x4 row address of this lane in the warp's 16-row Q tile
   const uint32_t qrow = (uint32_t)((warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * C::kRowBytes +
                                    ((lane >> 4) & 1) * 16);
-  const uint32_t qh_base = smem_u32(sQh) + qrow, ql_base = smem_u32(sQl) + qrow;
+  const uint32_t q_base = smem_u32(sQ) + qrow;
 
   if (c0 < c1) load_chunk<HD>(a, pt, pgs, pg0, kvh, c0, maxpos, smem, smem + C::kTileBytes, tid);
   for (int ch = c0; ch < c1; ++ch) {
     const int buf = (ch - c0) & 1;
-    const uint8_t* sK = smem + buf * 2 * C::kTileBytes;
-    const uint8_t* sV = sK + C::kTileBytes;
+    uint8_t* sK = smem + buf * 2 * C::kTileBytes;
+    uint8_t* sV = sK + C::kTileBytes;
     cp_async_wait_all();
+    chunk_to_f16<HD>(sK, sV, tid);
     bar();
     if (ch + 1 < c1) {
       uint8_t* nK = smem + (buf ^ 1) * 2 * C::kTileBytes;
@@ -206,21 +223,17 @@ __device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0
       for (int j = 0; j < NJ; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
 #pragma unroll
       for (int ks = 0; ks < KS; ++ks) {
-        uint32_t qh[4], ql[4], kb[NJ][2];
-        ldsm_x4(qh, qh_base + ks * 32);
-        ldsm_x4(ql, ql_base + ks * 32);
+        uint32_t qf[4], kb[NJ][2];
+        ldsm_x4(qf, q_base + ks * 32);
 #pragma unroll
         for (int j = 0; j < NJ; ++j) {
           const uint8_t* krow = sK + (j * 8 + g) * C::kRowBytes;
           kb[j][0] = *reinterpret_cast<const uint32_t*>(krow + (ks * 16 + 2 * c4) * 2);
           kb[j][1] = *reinterpret_cast<const uint32_t*>(krow + (ks * 16 + 8 + 2 * c4) * 2);
         }
-        // independent accumulators back to back; hi and lo products of one
-        // n-tile are NJ MMAs apart
+        // independent accumulators back to back
 #pragma unroll
-        for (int j = 0; j < NJ; ++j) mma_bf16_16816(s[j], qh, kb[j][0], kb[j][1]);
-#pragma unroll
-        for (int j = 0; j < NJ; ++j) mma_bf16_16816(s[j], ql, kb[j][0], kb[j][1]);
+        for (int j = 0; j < NJ; ++j) mma_f16_16816(s[j], qf, kb[j][0], kb[j][1]);
       }
       // scale, causal mask, online softmax (rows qa and qb)
       float mxa = -INFINITY, mxb = -INFINITY;
@@ -266,11 +279,11 @@ __device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0
       // O += P V: P as A fragments (keys are the k dimension), V via ldmatrix.trans
 #pragma unroll
       for (int kk = 0; kk < NJ / 2; ++kk) {
-        uint32_t ph[4], pl[4];
-        split2(s[2 * kk][0], s[2 * kk][1], ph[0], pl[0]);
-        split2(s[2 * kk][2], s[2 * kk][3], ph[1], pl[1]);
-        split2(s[2 * kk + 1][0], s[2 * kk + 1][1], ph[2], pl[2]);
-        split2(s[2 * kk + 1][2], s[2 * kk + 1][3], ph[3], pl[3]);
+        uint32_t pf[4];
+        pf[0] = pack_h2(s[2 * kk][0], s[2 * kk][1]);
+        pf[1] = pack_h2(s[2 * kk][2], s[2 * kk][3]);
+        pf[2] = pack_h2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+        pf[3] = pack_h2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
         const uint32_t vrow = smem_u32(sV + (kk * 16 + (lane & 15)) * C::kRowBytes);
 #pragma unroll
         for (int n0 = 0; n0 < NT; n0 += 4) {
@@ -278,9 +291,7 @@ __device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0
 #pragma unroll
           for (int u = 0; u < 4; ++u) ldsm_x2_trans(vb[u][0], vb[u][1], vrow + (n0 + u) * 16);
 #pragma unroll
-          for (int u = 0; u < 4; ++u) mma_bf16_16816(o[n0 + u], ph, vb[u][0], vb[u][1]);
-#pragma unroll
-          for (int u = 0; u < 4; ++u) mma_bf16_16816(o[n0 + u], pl, vb[u][0], vb[u][1]);
+          for (int u = 0; u < 4; ++u) mma_f16_16816(o[n0 + u], pf, vb[u][0], vb[u][1]);
         }
       }
     }
