@@ -351,8 +351,8 @@ AttnGeom attn_geometry(pard_ctx* c, int mi, int rows_per_seq, int batch) {
   AttnGeom g;
   g.row_blocks = (rows_per_seq + rb_rows - 1) / rb_rows;
   g.groups = batch * cf.n_kv_heads * g.row_blocks;
-  const int n_kt = (c->lim.max_ctx + 63) / 64;
-  g.n_split = std::max(1, std::min({8, n_kt, (2 * c->sm + g.groups - 1) / g.groups}));
+  const int n_kt = (c->lim.max_ctx + 31) / 32;  // 32-key chunks at the longest context
+  g.n_split = std::max(1, std::min({16, n_kt, (2 * c->sm + g.groups - 1) / g.groups}));
   return g;
 }
 
@@ -362,7 +362,7 @@ struct LayerPlan {
   AttnArgs at;
 };
 LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch, const int* pt_attn,
-                     const AttnGeom& geo) {
+                     const AttnGeom& geo, int fixed_rows) {
   Model& M = c->m[mi];
   const pard_model_cfg& cf = M.cfg;
   const int d = cf.d_model, qd = M.qd(), kvd = M.kvd(), ffn = cf.ffn;
@@ -400,7 +400,7 @@ LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch
     a.q = c->q; a.q_ld = qd;
     a.kcache = M.kcache(l); a.vcache = M.vcache(l);
     a.page_table = pt_attn; a.pt_ld = c->D.pt_ld;
-    a.row_pos = c->rp.row_pos; a.seq_row0 = c->rp.seq_row0; a.m_dev = c->rp.m_dev;
+    a.row_pos = c->rp.row_pos; a.seq_row0 = c->rp.seq_row0; a.rows_per_seq = fixed_rows; a.m_dev = c->rp.m_dev;
     a.batch = batch; a.hq = cf.n_q_heads; a.hkv = cf.n_kv_heads; a.hd = cf.head_dim;
     a.page_size = c->lim.page_size; a.n_pages = c->lim.n_pages;
     a.row_blocks = geo.row_blocks; a.n_split = geo.n_split;
@@ -461,11 +461,11 @@ LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch
 // decomposition; pt_attn: page table row base the attention kernel indexes
 // by its sequence index.
 void run_layers(pard_ctx* c, int mi, int rows_cap, int batch, int rows_per_seq, const int* pt_attn,
-                cudaStream_t s) {
+                cudaStream_t s, int fixed_rows = 0) {
   const int tt = pick_tt(rows_cap);
   const AttnGeom geo = attn_geometry(c, mi, rows_per_seq, batch);
   for (int l = 0; l < c->m[mi].cfg.n_layers; ++l) {
-    LayerPlan P = layer_plan(c, mi, l, rows_cap, tt, batch, pt_attn, geo);
+    LayerPlan P = layer_plan(c, mi, l, rows_cap, tt, batch, pt_attn, geo, fixed_rows);
     run_gemm(c, P.qkv, tt, s);
     launch_attention(P.at, geo.groups * geo.n_split, s, true);
     c->launches++;
@@ -550,7 +550,7 @@ void build_fwd(pard_ctx* c, int mi, int keep, cudaStream_t s) {
     ph.push_back(p);
   };
   for (int l = 0; l < M.cfg.n_layers; ++l) {
-    LayerPlan P = layer_plan(c, mi, l, rows_cap, kFwdTT, c->batch, M.page_table, geo);
+    LayerPlan P = layer_plan(c, mi, l, rows_cap, kFwdTT, c->batch, M.page_table, geo, draft ? 0 : c->K + 1);
     const int prev = (int)ph.size() - 1;  // -1 for the first layer: the embedding kernel precedes the launch
     gemm_phase(P.qkv, prev);
     Phase a;
@@ -1001,7 +1001,7 @@ pard_status pard_verify(pard_ctx* c, const int32_t* d_draft_in, float temperatur
     Model& M = c->m[0];
     const int keep = (c->last_draft_sampled || d_logits_out) ? 1 : 0;
     if (!try_fwd(c, 0, keep, s)) {
-      run_layers(c, 0, rows_cap, c->batch, c->K + 1, M.page_table, s);
+      run_layers(c, 0, rows_cap, c->batch, c->K + 1, M.page_table, s, c->K + 1);  // K + 1 rows per sequence
       const int tt = pick_tt(rows_cap);
       run_lm_head(c, 0, c->xd, 2 * c->D.MC, c->ssq, rows_cap, tt, c->rp.m_dev, keep ? c->logits : nullptr,
                   c->rp.row_out, nullptr, c->rp.row_seq, c->stats_t, c->stats_it, STREAM_BONUS, s);

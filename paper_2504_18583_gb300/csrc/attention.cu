@@ -20,83 +20,61 @@
 
 namespace pard {
 
+constexpr int kAttnBufs = 4;  // K/V chunk ring of the standalone kernel (3 chunks in flight)
+
 template <int HD, int GROUP>
 __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constant__ AttnArgs a) {
-  constexpr int RB = kMaxQV / GROUP;  // rows per block
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_pos[kMaxQV];
-  __shared__ float s_w[kMaxQV][kMaxCluster];
 
   pdl_wait();
-  pdl_trigger();  // the next kernel may start streaming its weights now
   const uint32_t rank = cluster_rank(), NS = cluster_size();
   const int group_idx = blockIdx.x / NS;
   const int rb = group_idx % a.row_blocks;
   const int kvh = (group_idx / a.row_blocks) % a.hkv;
   const int b = group_idx / (a.row_blocks * a.hkv);
-  const int M = *a.m_dev;
-  int row0 = 0, nrows = 0;
-  if (b < a.batch) {
-    row0 = a.seq_row0[b] + rb * RB;
-    int row_end = min(a.seq_row0[b + 1], row0 + RB);
-    row_end = min(row_end, M);
-    nrows = max(0, row_end - row0);
-  }
-  const int nqv = nrows * GROUP;
-  for (int r = threadIdx.x; r < kMaxQV; r += kAttnThreads) s_pos[r] = r < nrows ? a.row_pos[row0 + r] : -1;
-  __syncthreads();
-  int maxpos = -1;
-  for (int r = 0; r < nrows; ++r) maxpos = max(maxpos, s_pos[r]);
-  const int n_chunks = maxpos >= 0 ? maxpos / kKeyChunk + 1 : 0;
-  const int c0 = (int)((long)rank * n_chunks / NS), c1 = (int)((long)(rank + 1) * n_chunks / NS);
-  const int* pt = a.page_table + (size_t)(b < a.batch ? b : 0) * a.pt_ld;
-
-  attn_partial<HD, GROUP>(a, pt, kvh, row0, nrows, s_pos, maxpos, c0, c1, smem, threadIdx.x,
-                          [] { __syncthreads(); });
+  // with a fixed row count per sequence the row range needs no load
+  const int M = a.rows_per_seq > 0 ? a.batch * a.rows_per_seq : *a.m_dev;
+  const AttnRows R = attn_unit<HD, GROUP, kAttnBufs>(a, b, kvh, rb, (int)rank, (int)NS, M, smem, s_pos,
+                                                     threadIdx.x, [] { __syncthreads(); });
+  const int row0 = R.row0, nqv = R.nrows * GROUP;
+  // the next kernel may start streaming its weights once the key/value reads
+  // are done: earlier, its bulk loads would queue ahead of them
+  pdl_trigger();
   float* part = reinterpret_cast<float*>(smem);
   cluster_sync();
   // combine in rank order; CTA `rank` finishes query vectors rank, rank+NS, ...
-  // Every rank's value is requested before any is used (the loads overlap).
-  for (int qv = (int)rank + (int)NS * (int)threadIdx.x; qv < nqv; qv += (int)NS * kAttnThreads) {
-    float2 ml[kMaxCluster];
+  // Each thread takes one output pair (qv, d..d+1) at a time and requests
+  // every rank's (max, sum) and partial values before using any, so a round of
+  // work is one distributed-shared-memory round trip.
+  const int my_qv = nqv > (int)rank ? (nqv - (int)rank + (int)NS - 1) / (int)NS : 0;
+  const int n_items = my_qv * (HD / 2);
+  for (int i = threadIdx.x; i < n_items; i += kAttnThreads) {
+    const int qv = (int)rank + (int)NS * (i / (HD / 2)), d = 2 * (i % (HD / 2));
+    float2 ml[kMaxCluster], pv[kMaxCluster];
 #pragma unroll
-    for (int r = 0; r < kMaxCluster; ++r)
-      ml[r] = r < (int)NS ? ld_dsmem2(part + qv * (HD + 2) + HD, (uint32_t)r) : make_float2(-INFINITY, 0.f);
+    for (int r = 0; r < kMaxCluster; ++r) {
+      const bool live = r < (int)NS;
+      ml[r] = live ? ld_dsmem2(part + qv * (HD + 2) + HD, (uint32_t)r) : make_float2(-INFINITY, 0.f);
+      pv[r] = live ? ld_dsmem2(part + qv * (HD + 2) + d, (uint32_t)r) : make_float2(0.f, 0.f);
+    }
     float mx = -INFINITY;
 #pragma unroll
     for (int r = 0; r < kMaxCluster; ++r) mx = fmaxf(mx, ml[r].x);
-    float w[kMaxCluster], L = 0.f;
-#pragma unroll
-    for (int r = 0; r < kMaxCluster; ++r) {
-      w[r] = ml[r].x == -INFINITY ? 0.f : expf(ml[r].x - mx);
-      L += ml[r].y * w[r];
-    }
-#pragma unroll
-    for (int r = 0; r < kMaxCluster; ++r)
-      if (r < (int)NS) s_w[qv][r] = w[r] / L;
-  }
-  __syncthreads();
-  const int my_qv = nqv > (int)rank ? (nqv - (int)rank + (int)NS - 1) / (int)NS : 0;
-  for (int i = threadIdx.x; i < my_qv * (HD / 2); i += kAttnThreads) {
-    const int qv = (int)rank + (int)NS * (i / (HD / 2)), d = 2 * (i % (HD / 2));
-    float2 pv[kMaxCluster];
-#pragma unroll
-    for (int r = 0; r < kMaxCluster; ++r)
-      pv[r] = r < (int)NS ? ld_dsmem2(part + qv * (HD + 2) + d, (uint32_t)r) : make_float2(0.f, 0.f);
+    float L = 0.f;
     float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
     for (int r = 0; r < kMaxCluster; ++r) {
-      const float wr = r < (int)NS ? s_w[qv][r] : 0.f;
-      if (wr != 0.f) {
-        acc.x += pv[r].x * wr;
-        acc.y += pv[r].y * wr;
-      }
+      const float w = ml[r].x == -INFINITY ? 0.f : expf(ml[r].x - mx);
+      L += ml[r].y * w;
+      acc.x += pv[r].x * w;
+      acc.y += pv[r].y * w;
     }
     const int m = row0 + qv / GROUP;
     const int col = (kvh * GROUP + qv % GROUP) * HD + d;
     __nv_bfloat16 h0, l0, h1, l1;
-    split_bf16(acc.x, h0, l0);
-    split_bf16(acc.y, h1, l1);
+    split_bf16(acc.x / L, h0, l0);
+    split_bf16(acc.y / L, h1, l1);
     *reinterpret_cast<uint32_t*>(a.x_out + xpk(2 * m, col, a.x_rows)) =
         (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
     *reinterpret_cast<uint32_t*>(a.x_out + xpk(2 * m + 1, col, a.x_rows)) =
@@ -110,9 +88,11 @@ size_t attention_part_floats(int, int, int, int, int, int) { return 0; }
 template <int HD, int GROUP>
 static cudaError_t launch_attn_t(const AttnArgs& a, int grid, int cluster, cudaStream_t s, bool pdl) {
   static bool configured = false;
-  const int smem = AttnCfg<HD>::kSmem;
+  const int smem = AttnCfg<HD, kAttnBufs>::kSmem;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD, GROUP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(attn_kernel<HD, GROUP>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     configured = true;
   }
@@ -135,13 +115,25 @@ static cudaError_t launch_attn_t(const AttnArgs& a, int grid, int cluster, cudaS
 
 int attention_rows_per_block(int group) { return kMaxQV / group; }
 
-// grid = groups * n_split CTAs; the n_split (<= 8) CTAs of one cluster share
-// one (sequence, kv head, row block) and split its keys.
+// grid = groups * n_split CTAs; the n_split (<= 16) CTAs of one cluster share
+// one (sequence, kv head, row block) and split its keys.  A cluster above 8
+// CTAs that the GPU cannot place falls back to 8.
+static cudaError_t launch_attn_any(const AttnArgs& a, int group, int grid, int cl, cudaStream_t s, bool pdl);
+
 void launch_attention(const AttnArgs& a, int grid, cudaStream_t s, bool pdl) {
   const int group = a.hq / a.hkv;
   const int cl = a.n_split;
-  cudaError_t e = cudaErrorInvalidValue;
   if (cl < 1 || cl > kMaxCluster || grid % cl) throw cudaErrorInvalidValue;
+  cudaError_t e = launch_attn_any(a, group, grid, cl, s, pdl);
+  if (e != cudaSuccess && cl > 8) {
+    (void)cudaGetLastError();
+    e = launch_attn_any(a, group, grid / cl * 8, 8, s, pdl);
+  }
+  if (e != cudaSuccess) throw e;
+}
+
+static cudaError_t launch_attn_any(const AttnArgs& a, int group, int grid, int cl, cudaStream_t s, bool pdl) {
+  cudaError_t e = cudaErrorInvalidValue;
   if (a.hd == 128 && group == 4) e = launch_attn_t<128, 4>(a, grid, cl, s, pdl);
   else if (a.hd == 128 && group == 8) e = launch_attn_t<128, 8>(a, grid, cl, s, pdl);
   else if (a.hd == 64 && group == 4) e = launch_attn_t<64, 4>(a, grid, cl, s, pdl);
@@ -150,7 +142,7 @@ void launch_attention(const AttnArgs& a, int grid, cudaStream_t s, bool pdl) {
   else if (a.hd == 64 && group == 2) e = launch_attn_t<64, 2>(a, grid, cl, s, pdl);
   else if (a.hd == 128 && group == 1) e = launch_attn_t<128, 1>(a, grid, cl, s, pdl);
   else if (a.hd == 64 && group == 1) e = launch_attn_t<64, 1>(a, grid, cl, s, pdl);
-  if (e != cudaSuccess) throw e;
+  return e;
 }
 
 }  // namespace pard

@@ -14,17 +14,18 @@ namespace pard {
 constexpr int kAttnThreads = 128;  // 4 warps x 16 query vectors
 constexpr int kMaxQV = kMaxQVRows;
 constexpr int kKeyChunk = 32;
-constexpr int kMaxCluster = 8;
+constexpr int kMaxCluster = 16;  // key splits of one work unit (clusters above 8 are non-portable)
 constexpr int kAttnPageCache = 512;  // page ids of one work unit's key range held in shared memory
 
-// Shared memory of one work unit: K and V chunks double-buffered, Q as fp16
-// rows (the MMA A operand, read with ldmatrix), then the page id cache; the
-// partial result (o, m, l) reuses the front at the end.
-template <int HD>
+// Shared memory of one work unit: NBUF K/V chunk buffers (a ring, NBUF - 1
+// chunks in flight), Q as fp16 rows (the MMA A operand, read with ldmatrix),
+// then the page id cache; the partial result (o, m, l) reuses the front at the
+// end.
+template <int HD, int NBUF>
 struct AttnCfg {
   static constexpr int kRowBytes = HD * 2 + 16;             // padded smem row (conflict-free ldmatrix)
   static constexpr int kTileBytes = kKeyChunk * kRowBytes;  // one K or V chunk
-  static constexpr int kKV = 4 * kTileBytes;                // K and V, double-buffered
+  static constexpr int kKV = NBUF * 2 * kTileBytes;         // K and V chunk ring
   static constexpr int kQBytes = kMaxQV * kRowBytes;        // Q rows
   static constexpr int kQOff = kKV;
   static constexpr int kPart = kMaxQV * (HD + 2) * 4;       // partial (o, m, l) per CTA
@@ -85,24 +86,13 @@ __device__ __forceinline__ float2 ld_dsmem2(const float* local, uint32_t rank) {
   return v;
 }
 
-// Page id of the page holding key position pos (-1: none or invalid, flagged).
-__device__ __forceinline__ int page_of(const AttnArgs& a, const int* pt, int pos) {
-  int page = -1;
-  if (pos / a.page_size < a.pt_ld) page = pt[pos / a.page_size];
-  if (page < 0 || page >= a.n_pages) {
-    set_status(a.status, ST_BAD_PAGE);
-    page = -1;
-  }
-  return page;
-}
-
-// K and V rows of one 64-key chunk into shared memory; positions past maxpos
-// (masked anyway) and bad pages become zeros.  spg: page ids of the pages
-// pg0, pg0 + 1, ... (nullptr: read the page table here).
-template <int HD>
-__device__ __forceinline__ void load_chunk(const AttnArgs& a, const int* pt, const int* spg, int pg0, int kvh,
-                                           int chunk, int maxpos, uint8_t* sK, uint8_t* sV, int tid) {
-  using C = AttnCfg<HD>;
+// K and V rows of one 32-key chunk into shared memory; positions past maxpos
+// (masked anyway) and bad pages become zeros.  spg: the sequence's page table
+// row in shared memory (nullptr: read it from global memory here).
+template <int HD, int NBUF>
+__device__ __forceinline__ void load_chunk(const AttnArgs& a, const int* pt, const int* spg, int kvh, int chunk,
+                                           int maxpos, uint8_t* sK, uint8_t* sV, int tid) {
+  using C = AttnCfg<HD, NBUF>;
   constexpr int kCh = HD * 2 / 16;
   for (int i = tid; i < kKeyChunk * kCh; i += kAttnThreads) {
     const int key = i / kCh, ch = i % kCh;
@@ -110,7 +100,13 @@ __device__ __forceinline__ void load_chunk(const AttnArgs& a, const int* pt, con
     uint8_t* dk = sK + key * C::kRowBytes + ch * 16;
     uint8_t* dv = sV + key * C::kRowBytes + ch * 16;
     int page = -1;
-    if (pos <= maxpos) page = spg ? spg[pos / a.page_size - pg0] : page_of(a, pt, pos);
+    if (pos <= maxpos && pos / a.page_size < a.pt_ld) {
+      page = spg ? spg[pos / a.page_size] : pt[pos / a.page_size];
+      if (page < 0 || page >= a.n_pages) {
+        set_status(a.status, ST_BAD_PAGE);
+        page = -1;
+      }
+    }
     if (page < 0) {
       *reinterpret_cast<uint4*>(dk) = make_uint4(0, 0, 0, 0);
       *reinterpret_cast<uint4*>(dv) = make_uint4(0, 0, 0, 0);
@@ -120,14 +116,13 @@ __device__ __forceinline__ void load_chunk(const AttnArgs& a, const int* pt, con
     cp_async16(dk, a.kcache + off);
     cp_async16(dv, a.vcache + off);
   }
-  cp_async_commit();
 }
 
 // The same thread's pieces of a landed chunk (load_chunk's mapping), bf16 ->
 // fp16 in place; zero-filled pieces are zeros in both formats.
-template <int HD>
+template <int HD, int NBUF>
 __device__ __forceinline__ void chunk_to_f16(uint8_t* sK, uint8_t* sV, int tid) {
-  using C = AttnCfg<HD>;
+  using C = AttnCfg<HD, NBUF>;
   constexpr int kCh = HD * 2 / 16;
   for (int i = tid; i < kKeyChunk * kCh; i += kAttnThreads) {
     const int key = i / kCh, ch = i % kCh;
@@ -139,35 +134,72 @@ __device__ __forceinline__ void chunk_to_f16(uint8_t* sK, uint8_t* sV, int tid) 
   }
 }
 
-// Partial attention of 4 warps (tid 0..127, warp = tid / 32) over key chunks
-// [c0, c1): rows row0..row0+nrows-1 of the row block (positions in s_pos),
-// query vectors qv = r * GROUP + head.  Leaves the unnormalised output and the
-// softmax (max, sum) of each query vector in smem as [64][HD + 2] floats.
-// bar() synchronises the 128 threads.  Each warp writes its own query vectors'
-// entries on return; the caller synchronises before reading other warps'.
-template <int HD, int GROUP, typename Bar>
-__device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0, int nrows, const int* s_pos,
-                             int maxpos, int c0, int c1, uint8_t* smem, int tid, Bar bar) {
-  using C = AttnCfg<HD>;
+// Wait until at most n of this thread's most recent cp.async groups are pending.
+__device__ __forceinline__ void cp_async_wait_upto(int n) {
+  if (n <= 0) asm volatile("cp.async.wait_group 0;" ::: "memory");
+  else if (n == 1) asm volatile("cp.async.wait_group 1;" ::: "memory");
+  else asm volatile("cp.async.wait_group 2;" ::: "memory");
+}
+
+struct AttnRows {
+  int row0, nrows;
+};
+
+// One attention work unit of 4 warps (tid 0..127, warp = tid / 32): sequence
+// b, kv head kvh, row block rb (rows row0 .. row0 + nrows - 1 of the pass,
+// query vectors qv = r * GROUP + head), key split sp of ns over the 32-key
+// chunks up to the block's last position.  Leaves the unnormalised output and
+// the softmax (max, sum) of each query vector in smem as [64][HD + 2] floats
+// (each warp its own query vectors; the caller synchronises before reading
+// other warps'), and its row positions in s_pos[64].  bar() synchronises the
+// 128 threads.
+//
+// Latency structure: one round of loads brings the row positions, Q and the
+// sequence's page table row together; then NBUF - 1 chunks of K/V stay in
+// flight while the warps compute on the oldest.
+template <int HD, int GROUP, int NBUF, typename Bar>
+__device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp, int ns, int M, uint8_t* smem,
+                              int* s_pos, int tid, Bar bar) {
+  static_assert(NBUF >= 2 && NBUF <= 4, "chunk ring of 2 to 4 buffers");
+  using C = AttnCfg<HD, NBUF>;
+  constexpr int RB = kMaxQV / GROUP;  // rows per block
   constexpr int KS = HD / 16;
   constexpr int NT = HD / 8;
   constexpr int NJ = kKeyChunk / 8;  // 8-key n-tiles per chunk
   const int warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, c4 = lane & 3;
-  const int nqv = nrows * GROUP;
-  const int qa = warp * 16 + g, qb = qa + 8;
-  const int posa = qa < nqv ? s_pos[qa / GROUP] : -1, posb = qb < nqv ? s_pos[qb / GROUP] : -1;
-  uint8_t* sQ = smem + C::kQOff;
 
-  // Q into shared memory as fp16 rows (zeros past nqv); q is rewritten by every
-  // layer, by other CTAs of a persistent grid: L2 loads
-  constexpr int kQIter = kMaxQV * (HD / 4) / kAttnThreads;  // 8 or 16 float4 per thread
-  static_assert(kQIter % 4 == 0, "Q staging in groups of four");
-#pragma unroll 1
-  for (int i0 = 0; i0 < kQIter; i0 += 4) {
-    float4 v[4];
+  AttnRows R{0, 0};
+  if (b < a.batch) {
+    const int s0 = a.rows_per_seq > 0 ? b * a.rows_per_seq : a.seq_row0[b];
+    const int s1 = a.rows_per_seq > 0 ? s0 + a.rows_per_seq : a.seq_row0[b + 1];
+    R.row0 = s0 + rb * RB;
+    const int row_end = min(min(s1, R.row0 + RB), M);
+    R.nrows = max(0, row_end - R.row0);
+  }
+  const int row0 = R.row0, nrows = R.nrows;
+  const int nqv = nrows * GROUP;
+  const int* pt = a.page_table + (size_t)(b < a.batch ? b : 0) * a.pt_ld;
+  uint8_t* sQ = smem + C::kQOff;
+  int* spg = reinterpret_cast<int*>(smem + C::kPageOff);
+  const bool cached = a.pt_ld <= kAttnPageCache;
+
+  // ---- one round of loads: row positions, page table row, Q ----
+  const int pos_v = tid < nrows ? a.row_pos[row0 + tid] : -1;
+  int pg_v[kAttnPageCache / kAttnThreads];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+  for (int k = 0; k < kAttnPageCache / kAttnThreads; ++k) {
+    const int i = tid + k * kAttnThreads;
+    pg_v[k] = (cached && i < a.pt_ld) ? pt[i] : -1;
+  }
+  // q is rewritten by every layer, by other CTAs of a persistent grid: L2 loads
+  constexpr int kQIter = kMaxQV * (HD / 4) / kAttnThreads;  // 8 or 16 float4 per thread
+  constexpr int kQGroup = kQIter < 8 ? kQIter : 8;
+#pragma unroll 1
+  for (int i0 = 0; i0 < kQIter; i0 += kQGroup) {
+    float4 v[kQGroup];
+#pragma unroll
+    for (int u = 0; u < kQGroup; ++u) {
       const int i = tid + (i0 + u) * kAttnThreads;
       const int qv = i / (HD / 4), d4 = i % (HD / 4);
       v[u] = qv < nqv ? __ldcg(reinterpret_cast<const float4*>(a.q + (size_t)(row0 + qv / GROUP) * a.q_ld +
@@ -175,24 +207,34 @@ __device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0
                       : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < kQGroup; ++u) {
       const int i = tid + (i0 + u) * kAttnThreads;
       const int qv = i / (HD / 4), d4 = i % (HD / 4);
       *reinterpret_cast<uint2*>(sQ + qv * C::kRowBytes + d4 * 8) =
           make_uint2(pack_h2(v[u].x, v[u].y), pack_h2(v[u].z, v[u].w));
     }
   }
-
-  // page ids of the whole key range, one round of loads instead of one per key row
-  const int last = min(c1 * kKeyChunk - 1, maxpos);
-  const int pg0 = c0 * kKeyChunk / a.page_size;
-  const int npg = last >= c0 * kKeyChunk ? last / a.page_size + 1 - pg0 : 0;
-  int* spg = reinterpret_cast<int*>(smem + C::kPageOff);
-  const bool cached = npg <= kAttnPageCache;
-  if (cached)
-    for (int i = tid; i < npg; i += kAttnThreads) spg[i] = page_of(a, pt, (pg0 + i) * a.page_size);
+  if (tid < kMaxQV) s_pos[tid] = pos_v;
+#pragma unroll
+  for (int k = 0; k < kAttnPageCache / kAttnThreads; ++k) spg[tid + k * kAttnThreads] = pg_v[k];
   bar();
+  int maxpos = -1;
+  for (int r = 0; r < nrows; ++r) maxpos = max(maxpos, s_pos[r]);
+  const int n_chunks = maxpos >= 0 ? maxpos / kKeyChunk + 1 : 0;
+  const int c0 = (int)((long)sp * n_chunks / ns), c1 = (int)((long)(sp + 1) * n_chunks / ns);
+  const int n = c1 - c0;
   const int* pgs = cached ? spg : nullptr;
+  const int qa = warp * 16 + g, qb = qa + 8;
+  const int posa = qa < nqv ? s_pos[qa / GROUP] : -1, posb = qb < nqv ? s_pos[qb / GROUP] : -1;
+
+  // ---- K/V chunk ring: NBUF - 1 chunks in flight ----
+  auto kbuf = [&](int t) { return smem + (t % NBUF) * 2 * C::kTileBytes; };
+  int issued = 0;
+  for (; issued < n && issued < NBUF - 1; ++issued) {
+    uint8_t* k = kbuf(issued);
+    load_chunk<HD, NBUF>(a, pt, pgs, kvh, c0 + issued, maxpos, k, k + C::kTileBytes, tid);
+    cp_async_commit();
+  }
 
   float o[NT][4];
 #pragma unroll
@@ -200,21 +242,21 @@ __device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0
   float ma = -INFINITY, mb = -INFINITY, la = 0.f, lb = 0.f;
   const bool active = warp * 16 < nqv;
   // ldmatrix.x4 row address of this lane in the warp's 16-row Q tile
-  const uint32_t qrow = (uint32_t)((warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * C::kRowBytes +
-                                   ((lane >> 4) & 1) * 16);
-  const uint32_t q_base = smem_u32(sQ) + qrow;
+  const uint32_t q_base = smem_u32(sQ) + (uint32_t)((warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * C::kRowBytes +
+                                                    ((lane >> 4) & 1) * 16);
 
-  if (c0 < c1) load_chunk<HD>(a, pt, pgs, pg0, kvh, c0, maxpos, smem, smem + C::kTileBytes, tid);
-  for (int ch = c0; ch < c1; ++ch) {
-    const int buf = (ch - c0) & 1;
-    uint8_t* sK = smem + buf * 2 * C::kTileBytes;
+  for (int t = 0; t < n; ++t) {
+    const int ch = c0 + t;
+    uint8_t* sK = kbuf(t);
     uint8_t* sV = sK + C::kTileBytes;
-    cp_async_wait_all();
-    chunk_to_f16<HD>(sK, sV, tid);
+    cp_async_wait_upto(issued - 1 - t);  // chunk t has landed (this thread's copies)
+    chunk_to_f16<HD, NBUF>(sK, sV, tid);
     bar();
-    if (ch + 1 < c1) {
-      uint8_t* nK = smem + (buf ^ 1) * 2 * C::kTileBytes;
-      load_chunk<HD>(a, pt, pgs, pg0, kvh, ch + 1, maxpos, nK, nK + C::kTileBytes, tid);
+    if (issued < n) {  // refill the buffer every warp finished with (chunk t - 1)
+      uint8_t* k = kbuf(issued);
+      load_chunk<HD, NBUF>(a, pt, pgs, kvh, c0 + issued, maxpos, k, k + C::kTileBytes, tid);
+      cp_async_commit();
+      ++issued;
     }
     if (active) {
       // S = Q K^T for the chunk's keys: NJ n-tiles of 8 keys, Q fragments per k-step
@@ -316,6 +358,7 @@ __device__ void attn_partial(const AttnArgs& a, const int* pt, int kvh, int row0
       part[qb * (HD + 2) + HD + 1] = lb;
     }
   }
+  return R;
 }
 
 }  // namespace pard

@@ -34,7 +34,8 @@ template <int HD>
 struct FwdCfg {
   using Gm = GemmCfg<kFwdTT>;
   static constexpr int kRing = kFwdStages * Gm::kStageBytes;
-  static constexpr int kAttn = (AttnCfg<HD>::kSmem + 1023) / 1024 * 1024;
+  static constexpr int kAttnBufs = 3;  // K/V chunk ring (2 chunks in flight)
+  static constexpr int kAttn = (AttnCfg<HD, kAttnBufs>::kSmem + 1023) / 1024 * 1024;
   static constexpr int kPhase = (int)((sizeof(Phase) + 127) / 128 * 128);  // epilogue's copy of its phase
   static constexpr int kBar = 8 * (2 * kFwdStages + 5);  // full, empty, accf x2, acce x2, drain
   static constexpr int kMisc = 64;
@@ -187,7 +188,6 @@ __device__ __forceinline__ void store_pair4(__nv_bfloat16* x, int m, int col, in
 template <int HD, int GROUP>
 __global__ void __launch_bounds__(192, 1) fwd_kernel(const __grid_constant__ FwdArgs f) {
   constexpr int TT = kFwdTT, S = kFwdStages;
-  constexpr int RB = kMaxQV / GROUP;
   using C = GemmCfg<TT>;
   using F = FwdCfg<HD>;
   extern __shared__ uint8_t smem_raw[];
@@ -412,21 +412,9 @@ __global__ void __launch_bounds__(192, 1) fwd_kernel(const __grid_constant__ Fwd
           const int rb = gidx % at.row_blocks;
           const int kvh = (gidx / at.row_blocks) % at.hkv;
           const int b = gidx / (at.row_blocks * at.hkv);
-          int row0 = 0, nrows = 0;
-          if (b < at.batch) {
-            row0 = at.seq_row0[b] + rb * RB;
-            const int row_end = min(min(at.seq_row0[b + 1], row0 + RB), M);
-            nrows = max(0, row_end - row0);
-          }
-          const int nqv = nrows * GROUP;
-          for (int r = et; r < kMaxQV; r += 128) s_pos[r] = r < nrows ? at.row_pos[row0 + r] : -1;
-          epi_bar();
-          int maxpos = -1;
-          for (int r = 0; r < nrows; ++r) maxpos = max(maxpos, s_pos[r]);
-          const int n_chunks = maxpos >= 0 ? maxpos / kKeyChunk + 1 : 0;
-          const int c0 = (int)((long)sp * n_chunks / ns), c1 = (int)((long)(sp + 1) * n_chunks / ns);
-          const int* pt = at.page_table + (size_t)(b < at.batch ? b : 0) * at.pt_ld;
-          attn_partial<HD, GROUP>(at, pt, kvh, row0, nrows, s_pos, maxpos, c0, c1, sAttn, et, [] { epi_bar(); });
+          const AttnRows R = attn_unit<HD, GROUP, F::kAttnBufs>(at, b, kvh, rb, sp, ns, M, sAttn, s_pos, et,
+                                                                [] { epi_bar(); });
+          const int row0 = R.row0, nqv = R.nrows * GROUP;
           epi_bar();  // every warp's partial is in shared memory
           const float* part = reinterpret_cast<const float*>(sAttn);
           if (ns == 1) {

@@ -89,6 +89,7 @@ struct AttnArgs {
   int pt_ld;
   const int* row_pos;
   const int* seq_row0;        // [B+1] first row of each sequence in this pass
+  int rows_per_seq;           // > 0: every sequence has this many rows (row0 = b x it), seq_row0 unread
   const int* m_dev;
   int batch;
   int hq, hkv, hd, page_size, n_pages;
