@@ -97,9 +97,78 @@ __device__ __forceinline__ void store_pair8(__nv_bfloat16* x, int m, int col, in
   *reinterpret_cast<uint4*>(x + xpk(2 * m + 1, col, x_rows)) = make_uint4(l[0], l[1], l[2], l[3]);
 }
 
-// One 16-token chunk of the epilogue for the thread holding weight row fr.
+// Loads of one 16-token chunk's epilogue that do not depend on the tile's
+// result: the residual and norm gains (O / down), the row's position, KV page
+// and RoPE factors (QKV), the rows' output facts (LM head).  Taken before the
+// split-K arrival, so that the CTA that finishes a tile has them in hand.
+struct EpiPre {
+  uint4 w[8];     // O / down: h (w[0..3] as float4) and g (w[4..5]); QKV: 16 (cos, sin) pairs
+  int pos, page;  // QKV: position (-1 invalid) and KV page (-1 none) of the thread's token
+  int ri[3];      // LM head, threads et < 16: logits row, Gumbel index, sequence of token et
+  int ok;         // O / down: the vector loads above were taken
+};
+
+static __device__ __forceinline__ EpiPre epi_pre(const GemmArgs& a, int w_tile, int tok0, int et, int M) {
+  EpiPre p;
+  p.ok = 0;
+  p.pos = -1;
+  p.page = -1;
+  const int jl = et >> 3, c16 = (et & 7) * 16;
+  const int mr = tok0 + jl;
+  if (a.mode == MODE_RESID) {
+    const int n0 = w_tile * kTileN + c16;
+    if (mr < M && n0 + 16 <= a.seg_rows[0] && (reinterpret_cast<uintptr_t>(a.g_next) & 15) == 0) {
+      // L2: other CTAs of a persistent grid update h
+      const float4* hp = reinterpret_cast<const float4*>(a.h + (size_t)mr * a.h_ld + n0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float4 h = __ldcg(hp + i);
+        p.w[i] = make_uint4(__float_as_uint(h.x), __float_as_uint(h.y), __float_as_uint(h.z), __float_as_uint(h.w));
+      }
+#pragma unroll
+      for (int i = 0; i < 2; ++i) p.w[4 + i] = *reinterpret_cast<const uint4*>(a.g_next + n0 + 8 * i);
+      p.ok = 1;
+    }
+  } else if (a.mode == MODE_QKV) {
+    const int seg = seg_of(a, w_tile);
+    const int n0 = (w_tile - a.seg_tile0[seg]) * kTileN + c16;
+    if (mr < M) {
+      const int pos = a.row_pos[mr];
+      const bool pv = pos >= 0 && pos / a.page_size < a.pt_ld;
+      if (!pv && (et & 7) == 0) set_status(a.status, ST_BAD_POS);
+      if (pv) {
+        p.pos = pos;
+        if (seg > 0) {
+          const int page = a.page_table[(size_t)a.row_seq[mr] * a.pt_ld + pos / a.page_size];
+          if (page >= 0 && page < a.n_pages) p.page = page;
+          else if ((et & 7) == 0) set_status(a.status, ST_BAD_PAGE);
+        }
+        if (seg < 2 && n0 < a.seg_rows[seg]) {
+          const int half = a.hd >> 1, jj = n0 % a.hd;
+          const int fi0 = jj < half ? jj : jj - half;
+          const uint4* csp = reinterpret_cast<const uint4*>(a.rope + (size_t)pos * half + fi0);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) p.w[i] = csp[i];
+        }
+      }
+    }
+  } else if (a.mode == MODE_LOGITS) {
+    if (et < kEpiTok) {
+      const int m = tok0 + et;
+      const bool in = m < M;
+      const bool sample = a.call->sample != 0 && a.row_gi != nullptr;
+      p.ri[0] = in ? (a.row_out ? a.row_out[m] : m) : -1;
+      p.ri[1] = (in && sample) ? a.row_gi[m] : -1;
+      p.ri[2] = (in && sample) ? a.row_seq[m] : 0;
+    }
+  }
+  return p;
+}
+
+// One 16-token chunk of the epilogue for the thread holding weight row fr;
+// pre holds the chunk's result-independent loads (epi_pre).
 static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_tile, int tok0, int rs_off, int fr,
-                          int et, int M, const EpiSmem& S) {
+                          int et, int M, const EpiSmem& S, const EpiPre& pre) {
   const int q = fr >> 5, lane = fr & 31;
   if (a.ssq_in) {
 #pragma unroll
@@ -120,15 +189,15 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
     if (mr < M && n0 < a.seg_rows[0]) {
       const float* xv = S.xch + jl * kTileN + c16;
       float* hp = a.h + (size_t)mr * a.h_ld + n0;
-      if (n0 + 16 <= a.seg_rows[0] && (reinterpret_cast<uintptr_t>(a.g_next) & 15) == 0) {
-        // every load first (one round trip; L2: other CTAs of a persistent
-        // grid update h), then the stores
+      if (pre.ok) {
         float4 hv[4];
         uint4 gv[2];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) hv[i] = __ldcg(reinterpret_cast<const float4*>(hp) + i);
+        for (int i = 0; i < 4; ++i)
+          hv[i] = make_float4(__uint_as_float(pre.w[i].x), __uint_as_float(pre.w[i].y), __uint_as_float(pre.w[i].z),
+                              __uint_as_float(pre.w[i].w));
 #pragma unroll
-        for (int i = 0; i < 2; ++i) gv[i] = *reinterpret_cast<const uint4*>(a.g_next + n0 + 8 * i);
+        for (int i = 0; i < 2; ++i) gv[i] = pre.w[4 + i];
         float hn[16];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -168,31 +237,11 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
     epi_bar();  // S.xch is rewritten by the next chunk
   } else if (a.mode == MODE_QKV) {
     const int seg = seg_of(a, w_tile);
-    // row facts of the chunk: position (-1: invalid) and KV page (-1: none)
-    if (et < kEpiTok) {
-      const int m = tok0 + et;
-      int pos = -1, page = -1;
-      if (m < M) {
-        pos = a.row_pos[m];
-        if (pos < 0 || pos / a.page_size >= a.pt_ld) {
-          set_status(a.status, ST_BAD_POS);
-          pos = -1;
-        } else if (seg > 0) {
-          page = a.page_table[(size_t)a.row_seq[m] * a.pt_ld + pos / a.page_size];
-          if (page < 0 || page >= a.n_pages) {
-            set_status(a.status, ST_BAD_PAGE);
-            page = -1;
-          }
-        }
-      }
-      S.ri[et] = pos;
-      S.ri[kEpiTok + et] = page;
-    }
 #pragma unroll
     for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
     epi_bar();
     const int n0 = (w_tile - a.seg_tile0[seg]) * kTileN + c16;  // first column within the segment
-    const int pos = S.ri[jl];
+    const int pos = pre.pos;
     if (mr < M && n0 < a.seg_rows[seg] && pos >= 0) {
       const float* xv = S.xch + jl * kTileN;
       float o[16];
@@ -203,12 +252,12 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
         // partner half of that head is in the same 128-row tile
         const int half = a.hd >> 1, jj = n0 % a.hd;
         const bool lo_half = jj < half;
-        const int fi0 = lo_half ? jj : jj - half;
         const int pc = lo_half ? c16 + half : c16 - half;
-        const float4* csp = reinterpret_cast<const float4*>(a.rope + (size_t)pos * half + fi0);
-        float4 cs4[8];
+        float4 cs4[8];  // 16 (cos, sin) pairs
 #pragma unroll
-        for (int i = 0; i < 8; ++i) cs4[i] = csp[i];  // 16 (cos, sin) pairs
+        for (int i = 0; i < 8; ++i)
+          cs4[i] = make_float4(__uint_as_float(pre.w[i].x), __uint_as_float(pre.w[i].y), __uint_as_float(pre.w[i].z),
+                               __uint_as_float(pre.w[i].w));
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const float c = (i & 1) ? cs4[i >> 1].z : cs4[i >> 1].x;
@@ -222,7 +271,7 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
 #pragma unroll
         for (int i = 0; i < 4; ++i) qp[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
       } else {
-        const int page = S.ri[kEpiTok + jl];
+        const int page = pre.page;
         if (page >= 0) {
           const int kvh = n0 / a.hd, e0 = n0 % a.hd;
           __nv_bfloat16* base = seg == 1 ? a.kcache : a.vcache;
@@ -238,7 +287,7 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
         }
       }
     }
-    epi_bar();  // S.xch and the row facts are rewritten by the next chunk
+    epi_bar();  // S.xch is rewritten by the next chunk
   } else if (a.mode == MODE_SWIGLU) {
 #pragma unroll
     for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
@@ -274,11 +323,9 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
     const bool sample = a.call->sample != 0 && a.row_gi != nullptr;
     // row facts of the chunk: logits row (-1: none), Gumbel index (-1: none), sequence
     if (et < kEpiTok) {
-      const int m = tok0 + et;
-      const bool in = m < M;
-      S.ri[et] = in ? (a.row_out ? a.row_out[m] : m) : -1;
-      S.ri[kEpiTok + et] = (in && sample) ? a.row_gi[m] : -1;
-      S.ri[2 * kEpiTok + et] = (in && sample) ? a.row_seq[m] : 0;
+      S.ri[et] = pre.ri[0];
+      S.ri[kEpiTok + et] = pre.ri[1];
+      S.ri[2 * kEpiTok + et] = pre.ri[2];
     }
     epi_bar();
     float x[kEpiTok];
@@ -374,7 +421,8 @@ __device__ void epi_segment(const GemmArgs& a, long t, long ub, long ue, long u0
       float v[kEpiTok];
 #pragma unroll
       for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
-      epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S);
+      epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S,
+                epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M));
     }
   } else {
     const int slot = (ub == u0) ? 0 : 1;
@@ -391,6 +439,9 @@ __device__ void epi_segment(const GemmArgs& a, long t, long ub, long ue, long u0
                               __uint_as_float(r[8 * j4 + 4]) + __uint_as_float(r[8 * j4 + 5]),
                               __uint_as_float(r[8 * j4 + 6]) + __uint_as_float(r[8 * j4 + 7]));
     }
+    // the result-independent loads of the finishing epilogue go out now, so
+    // the CTA that turns out to finish the tile does not wait for them
+    const EpiPre pre0 = epi_pre(a, w_tile, tok_base, et, M);
     // the barrier orders every thread's partial before the one acq_rel
     // arrival (cumulative), which also acquires the earlier arrivals' partials
     epi_bar();
@@ -408,11 +459,11 @@ __device__ void epi_segment(const GemmArgs& a, long t, long ub, long ue, long u0
         float v[kEpiTok];
 #pragma unroll
         for (int j = 0; j < kEpiTok; ++j) v[j] = 0.f;
-        // contributors in CTA order, four partial tiles requested per round trip
-        for (long cc0 = cf; cc0 <= cl; cc0 += 4) {
-          float4 pv[4][4];
+        // contributors in CTA order, two partial tiles requested per round trip
+        for (long cc0 = cf; cc0 <= cl; cc0 += 2) {
+          float4 pv[2][4];
 #pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4) {
+          for (int q4 = 0; q4 < 2; ++q4) {
             const long cc = cc0 + q4;
             if (cc <= cl && cc != c) {
               const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
@@ -423,7 +474,7 @@ __device__ void epi_segment(const GemmArgs& a, long t, long ub, long ue, long u0
             }
           }
 #pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4) {
+          for (int q4 = 0; q4 < 2; ++q4) {
             const long cc = cc0 + q4;
             if (cc > cl) break;
             if (cc == c) {
@@ -440,7 +491,8 @@ __device__ void epi_segment(const GemmArgs& a, long t, long ub, long ue, long u0
             }
           }
         }
-        epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S);
+        epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S,
+                  ch == 0 ? pre0 : epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M));
       }
       if (et == 0) a.counters[t] = 0;
     }
