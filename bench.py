@@ -44,6 +44,30 @@ def peaks():
     return 6800.0, "fallback"
 
 
+def kernel_source_hash() -> str:
+    """Hash of the CUDA sources and the C header (ties a measured traffic figure to the code it was taken on)."""
+    import glob
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2504_18583_gb300", "csrc")
+    files = sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh")) +
+                   glob.glob(os.path.join(csrc, "*.h")) + [os.path.join(ROOT, "include", "pard.h")])
+    for f in files:
+        h.update(os.path.basename(f).encode())
+        h.update(open(f, "rb").read())
+    return h.hexdigest()[:16]
+
+
+def measured_verify_traffic(persistent: bool):
+    """DRAM bytes of one verify pass from the committed ncu summary, or None when
+    the kernels changed since it was taken (or the pass runs another kernel)."""
+    p = os.path.join(ROOT, "profiles", "verify_pass_dram_traffic_8b.json")
+    if persistent or not os.path.exists(p):
+        return None
+    d = json.load(open(p))
+    return d["verify_traffic_bytes"] if d.get("csrc_sha") == kernel_source_hash() else None
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle sampling during the timed region."""
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -364,7 +388,10 @@ def main():
                      "kernel": ("verify pass: embedding kernel + one persistent fwd_kernel launch" if fused_used
                                 else "verify pass (all its launches; GEMM-dominated)"),
                      "achieved": ver_gbs, "peak": peak, "unit": "GB/s", "frac": ver_gbs / peak,
-                     "peak_kind": peak_kind, "traffic": None, "bytes_per_launch": vb,
+                     "peak_kind": peak_kind, "traffic": None if args.layers else measured_verify_traffic(fused_used),
+                     "traffic_source": "profiles/verify_pass_dram_traffic_8b.json (ncu DRAM bytes, 2-layer capture "
+                                       "scaled to 32 layers; null if the kernels changed since)",
+                     "bytes_per_launch": vb,
                      "bytes_note": "target weights 15.01 GB + KV read over the context + K+1 rows of KV written"},
         "phases_ms": {"draft": dr_ms, "verify": ver_ms, "accept": acc_ms},
         "draft_roofline": {"achieved": dr_gbs, "frac": dr_gbs / peak, "bytes": db},
