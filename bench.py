@@ -355,6 +355,56 @@ def main():
 
     e2e_tps, e2e_steps, prompt_bytes = e2e_run() if not args.no_e2e else (None, 1, 0)
 
+    # planted acceptance: the verify input is the target's own greedy
+    # continuation with each candidate corrupted with probability 1 - alpha, so
+    # the accepted prefix follows the rate the paper reports for a trained PARD
+    # draft; the draft pass still runs every step (T_step = T_draft + T_verify)
+    def planted_run(alpha: float, n_steps: int, seed: int = 7):
+        first = eng.prefill(prompts, wl.n_new, wl.K)
+        out = eng.alloc_step_outputs()
+        cont = [int(first[0])]
+        s = 0
+        while len(cont) < wl.n_new:
+            s += 1
+            eng.step(out, step=s)
+            k = int(out["n_emit"][0])
+            cont += [int(t) for t in out["emitted"][0][:k].tolist()]
+        rng = np.random.default_rng(seed)
+        plan, g = [], 1
+        while len(plan) < n_steps and g + wl.K <= len(cont):
+            cand = np.array(cont[g:g + wl.K], dtype=np.int32)
+            bad = rng.random(wl.K) >= alpha
+            cand[bad] = (cand[bad] + 1) % (wl.target.vocab - 1)
+            a = int(np.argmax(bad)) if bad.any() else wl.K
+            plan.append((cand, a))
+            g += a + 1
+        cands = torch.as_tensor(np.stack([c for c, _ in plan])[:, None, :], device="cuda")
+        eng.prefill(prompts, wl.n_new, wl.K)
+        out = eng.alloc_step_outputs()
+        n_emit = torch.zeros(len(plan), dtype=torch.int32, device="cuda")
+        acc = torch.zeros(len(plan), dtype=torch.int32, device="cuda")
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(len(plan)):
+            eng.draft(out, False, 1.0, 0, i + 1)
+            eng.verify(out, cands[i], 1.0)
+            eng.accept_commit(out, False, 1.0, 0, i + 1)
+            n_emit[i:i + 1].copy_(out["n_emit"][:1])
+            acc[i:i + 1].copy_(out["accept_len"][:1])
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        toks = int(n_emit.sum().item())
+        return {"alpha": alpha, "steps": len(plan), "value": toks / (ms / 1e3), "unit": "tokens/s",
+                "ms_per_step": ms / len(plan), "tokens_per_step": toks / len(plan),
+                "accepted_per_step": float(acc.float().mean().item()),
+                "planned_accepted_per_step": float(np.mean([a for _, a in plan])),
+                "note": "verify input = the target's greedy continuation with each candidate corrupted "
+                        "with probability 1 - alpha (seeded); draft still runs every step"}
+
+    planted = planted_run(0.90, 24) if not args.layers else None
+
     # roofline of the verify pass
     peak, peak_kind = peaks()
     ver_ms = statistics.median(phases["verify"])
@@ -395,6 +445,7 @@ def main():
                      "bytes_note": "target weights 15.01 GB + KV read over the context + K+1 rows of KV written"},
         "phases_ms": {"draft": dr_ms, "verify": ver_ms, "accept": acc_ms},
         "draft_roofline": {"achieved": dr_gbs, "frac": dr_gbs / peak, "bytes": db},
+        "planted_acceptance": planted,
         "projection": {"alpha": alpha, "tokens_per_step": tok_per_step_proj,
                        "tokens_per_s": tok_per_step_proj / (step_ms / 1e3),
                        "note": "acceptance rate from the paper (context); same measured step time"},
