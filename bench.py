@@ -405,6 +405,31 @@ def main():
 
     planted = planted_run(0.90, 24) if not args.layers else None
 
+    # autoregressive baseline on the same kernels: the target alone, one token
+    # per verify + accept (K = 0), the decoding the paper's speedups are against
+    def ar_run(n_steps: int, warm: int = 3):
+        eng.prefill(prompts, wl.n_new, 0)
+        out = eng.alloc_step_outputs()
+        for i in range(warm):
+            eng.step(out, step=i + 1)
+        n_emit = torch.zeros(n_steps, dtype=torch.int32, device="cuda")
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(n_steps):
+            eng.step(out, step=warm + i + 1)
+            n_emit[i:i + 1].copy_(out["n_emit"][:1])
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        toks = int(n_emit.sum().item())
+        return {"value": toks / (ms / 1e3), "unit": "tokens/s", "ms_per_token": ms / max(toks, 1), "steps": n_steps,
+                "note": "target alone, one token per step (pard_prefill K = 0: verify + accept, no draft)"}
+
+    ar = ar_run(30) if not args.layers else None
+    if planted and ar:
+        planted["speedup_vs_autoregressive"] = planted["value"] / ar["value"]
+
     # roofline of the verify pass
     peak, peak_kind = peaks()
     ver_ms = statistics.median(phases["verify"])
@@ -446,6 +471,7 @@ def main():
         "phases_ms": {"draft": dr_ms, "verify": ver_ms, "accept": acc_ms},
         "draft_roofline": {"achieved": dr_gbs, "frac": dr_gbs / peak, "bytes": db},
         "planted_acceptance": planted,
+        "autoregressive_baseline": ar,
         "projection": {"alpha": alpha, "tokens_per_step": tok_per_step_proj,
                        "tokens_per_s": tok_per_step_proj / (step_ms / 1e3),
                        "note": "acceptance rate from the paper (context); same measured step time"},

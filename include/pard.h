@@ -114,7 +114,11 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* target, cons
  * Reserves ceil((len + n_new + 2K) / page_size) pages per sequence and
  * model, in sequence order, from the front of the page order.
  * n_new: tokens to generate per sequence, the first one included; K: the
- * draft length every later pard_draft uses.  Synchronises `stream`. */
+ * draft length every later pard_draft uses.  K = 0 selects autoregressive
+ * decoding with the target alone (Eq. 2): each pard_verify runs one row per
+ * sequence and pard_accept_commit emits its argmax (or a draw from it), and
+ * pard_draft returns PARD_ERR_STATE; it is the baseline the paper's speedups
+ * are measured against.  Synchronises `stream`. */
 pard_status pard_prefill(pard_ctx* ctx, const int32_t* d_tokens, const int32_t* h_lens, int32_t batch,
                          int32_t n_new, int32_t K, int32_t sample, float temperature, uint64_t seed,
                          int32_t* d_first_token, void* stream);

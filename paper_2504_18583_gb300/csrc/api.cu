@@ -532,7 +532,7 @@ void build_fwd(pard_ctx* c, int mi, int keep, cudaStream_t s) {
   const bool draft = mi == 1;
   const int rows_per_seq = draft ? 2 * c->K : c->K + 1;
   const int rows_cap = c->batch * rows_per_seq;
-  if (!c->fwd_enabled || rows_cap > kFwdTT || !fwd_shape_ok(M)) return;
+  if (!c->fwd_enabled || rows_cap == 0 || rows_cap > kFwdTT || !fwd_shape_ok(M)) return;
   if (5 * M.cfg.n_layers + 1 > c->D.fwd_phases) return;
   AttnGeom geo = attn_geometry(c, mi, rows_per_seq, c->batch);
   // one CTA per SM runs the attention items (group, split) = c, c + grid, ...
@@ -859,7 +859,7 @@ pard_status pard_prefill(pard_ctx* c, const int32_t* d_tokens, const int32_t* h_
   if (!c || !d_tokens || !h_lens || !d_first) return fail(PARD_ERR_ARG, "null argument");
   if (c->unpacked) return fail(PARD_ERR_STATE, "weights were unpacked; load them again");
   if (batch < 1 || batch > c->lim.max_batch) return fail(PARD_ERR_ARG, "batch outside [1, max_batch]");
-  if (K < 1 || K > c->lim.max_k) return fail(PARD_ERR_ARG, "K outside [1, max_k]");
+  if (K < 0 || K > c->lim.max_k) return fail(PARD_ERR_ARG, "K outside [0, max_k]");
   if (n_new < 1) return fail(PARD_ERR_ARG, "n_new < 1");
   if (sample && !(temperature > 0.f)) return fail(PARD_ERR_ARG, "temperature must be > 0 when sampling");
   const int ps = c->lim.page_size;
@@ -947,6 +947,7 @@ pard_status pard_draft(pard_ctx* c, int32_t sample, float temperature, uint64_t 
                        float* d_logits, void* stream) {
   if (!c) return fail(PARD_ERR_ARG, "null context");
   if (!c->prefilled) return fail(PARD_ERR_STATE, "pard_draft before pard_prefill (or after pard_unpack_weights)");
+  if (c->K == 0) return fail(PARD_ERR_STATE, "pard_draft with K = 0 (autoregressive decoding has no draft pass)");
   if (sample && !(temperature > 0.f)) return fail(PARD_ERR_ARG, "temperature must be > 0 when sampling");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   c->launches = 0;
@@ -999,7 +1000,8 @@ pard_status pard_verify(pard_ctx* c, const int32_t* d_draft_in, float temperatur
     launch_embed(e, rows_cap, s, true);
     c->launches++;
     Model& M = c->m[0];
-    const int keep = (c->last_draft_sampled || d_logits_out) ? 1 : 0;
+    // K = 0 (autoregressive) keeps its single row of logits for a sampled accept
+    const int keep = (c->last_draft_sampled || d_logits_out || c->K == 0) ? 1 : 0;
     if (!try_fwd(c, 0, keep, s)) {
       run_layers(c, 0, rows_cap, c->batch, c->K + 1, M.page_table, s, c->K + 1);  // K + 1 rows per sequence
       const int tt = pick_tt(rows_cap);

@@ -225,8 +225,9 @@ class PardEngine:
                                         self.stream.cuda_stream), "pard_accept_commit")
 
     def step(self, out, sample=False, temperature=1.0, seed=0, step=0):
-        """One PARD step: draft, verify, accept/commit."""
-        self.draft(out, sample, temperature, seed, step)
+        """One PARD step: draft, verify, accept/commit (K = 0: one autoregressive token, no draft)."""
+        if self.K:
+            self.draft(out, sample, temperature, seed, step)
         self.verify(out, None, temperature)
         self.accept_commit(out, sample, temperature, seed, step)
 

@@ -135,6 +135,43 @@ def test_full_width_8b_layers_short_prompt(fused):
     print("stats", P.stats)
 
 
+def test_autoregressive_mode_k0_matches_the_oracle_forward():
+    """K = 0: each pard_verify + pard_accept_commit decodes one token with the
+    target alone (Eq. 2); logits and tokens against one oracle forward per
+    token, teacher-forced onto the GPU's token."""
+    from paper_2504_18583_gb300 import pard
+    wl = S.WORKLOADS["tiny"].replace(n_new=20)
+    tw = S.model_weights(wl.target, wl.seed, S.TARGET, wl.norm_jitter)
+    dw = S.model_weights(wl.draft, wl.seed, S.DRAFT, wl.norm_jitter)
+    prompt = [int(t) for t in wl.prompts()[0]]
+    P_len = len(prompt)
+    eng = pard.PardEngine(wl.target, S.device_weights(wl.target, 0, 0, host=tw), wl.draft,
+                          S.device_weights(wl.draft, 0, 0, host=dw), max_batch=1, max_k=wl.K,
+                          max_ctx=P_len + wl.n_new + 2 * wl.K + 16, n_pages=wl.n_pages(), prefill_chunk=64,
+                          page_order_target=wl.page_order(S.TARGET), page_order_draft=wl.page_order(S.DRAFT))
+    stats = dict(excused_tokens=0, checked_tokens=0)
+    m = oracle.OracleModel(wl.target, tw, 1, P_len + wl.n_new + 2)
+    lg = m.forward(0, prompt, np.arange(P_len, dtype=np.int32), [P_len - 1])[0]
+    tok = int(eng.prefill([prompt], wl.n_new, 0).cpu().numpy()[0])
+    check_token(tok, lg, stats, "first token")
+    out = eng.alloc_step_outputs(want_logits=True)
+    for step in range(1, wl.n_new):
+        eng.verify(out, None, 1.0)
+        y = out["logits"][0, 0].cpu().numpy()
+        lg = m.forward(0, [tok], [P_len + step - 1], [0])[0]
+        assert float(np.abs(y - lg).max()) <= LOGIT_TOL, f"step {step}"
+        eng.accept_commit(out, False, 1.0, 0, step)
+        assert int(out["n_emit"][0]) == 1 and int(out["accept_len"][0]) == 0
+        tok = int(out["emitted"][0, 0])
+        check_token(tok, lg, stats, f"step {step}")
+    n, gen, done = eng.state()
+    assert gen == [wl.n_new] and done == [1]
+    assert eng.last_status() == 0
+    with pytest.raises(RuntimeError):
+        eng.draft(out)
+    print("stats", stats)
+
+
 # ----------------------------------------------------------------------------
 # speculative sampling
 # ----------------------------------------------------------------------------
