@@ -34,6 +34,12 @@ METRIC = "generated tokens/s (batch 1, 8B-shaped) + verify-step HBM GB/s as % of
 WORKLOAD_DESC = ("LLaMA3.1-8B-shaped target (32 layers, d 4096, 32q/8kv heads, ffn 14336, vocab 128256) + "
                  "LLaMA3.2-1B-shaped PARD draft (16 layers, d 2048), batch 1, 512-token prompt, K=8, greedy, "
                  "256 new tokens, KV page 16")
+WORKLOAD_DESCS = {
+    "8b_greedy": WORKLOAD_DESC,
+    "8b_sample": WORKLOAD_DESC.replace("512-token prompt, K=8, greedy", "1024-token prompt, K=6, speculative sampling T=1"),
+    "8b_batch16": WORKLOAD_DESC.replace("batch 1, 512-token prompt, K=8, greedy, 256 new tokens",
+                                        "batch 16, ragged prompts U[128, 2048], K=6, greedy, 128 new tokens"),
+}
 
 
 def peaks():
@@ -126,13 +132,13 @@ def dist_env():
 
 def verify_bytes(wl, ctx_tokens: float) -> float:
     """Algorithmic HBM bytes of one verify pass: every target weight once
-    (layers, norms, LM head), the KV cache read over the context, the K+1
-    new rows' K/V written, and the logits statistics (not the logits, which
-    the greedy path does not store)."""
+    (layers, norms, LM head), the KV cache read over the context (ctx_tokens:
+    summed over the batch), the K+1 new rows' K/V written per sequence; the
+    logits statistics are negligible (the greedy path stores no logits)."""
     t = wl.target
     kv_tok = t.kv_bytes_per_token()
     w = t.streamed_weight_bytes()
-    rows = wl.K + 1
+    rows = wl.batch * (wl.K + 1)
     return w + ctx_tokens * kv_tok + rows * kv_tok
 
 
@@ -224,6 +230,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end generation (profiling runs)")
     ap.add_argument("--persistent", action="store_true",
                     help="run draft / verify as one persistent kernel instead of one kernel per phase")
+    ap.add_argument("--workload", default="8b_greedy", choices=["8b_greedy", "8b_sample", "8b_batch16"],
+                    help="8b_greedy (the headline), 8b_sample (T = 1, K = 6), 8b_batch16 (16 ragged prompts, K = 6)")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling aid: truncate both models to this many layers (not a bench number)")
     args = ap.parse_args()
@@ -243,12 +251,12 @@ def main():
         dist.init_process_group("nccl")
     _build.build()
 
-    wl = S.WORKLOADS["8b_greedy"]
+    wl = S.WORKLOADS[args.workload]
     if args.layers:
         wl = wl.replace(target=wl.target.replace(n_layers=args.layers),
                         draft=wl.draft.replace(n_layers=min(args.layers, wl.draft.n_layers)))
     if args.warmup + args.steps > wl.n_new - 2:
-        raise SystemExit("warmup + steps must stay below the generation length (256)")
+        raise SystemExit(f"warmup + steps must stay below the generation length ({wl.n_new})")
     keep_host = rank == 0 and not args.no_cpu_baseline
     t_gen = time.perf_counter()
     host_t = S.model_weights(wl.target, wl.seed, S.TARGET) if keep_host else None
@@ -265,37 +273,39 @@ def main():
     eng.set_fused_pass(args.persistent)
     stream = eng.stream
 
+    sample, temp, seed = wl.sample, wl.temperature, 1
+
     def generation(timed_steps: int, warmup: int, phase_events: bool):
-        eng.prefill(prompts, wl.n_new, wl.K)
+        eng.prefill(prompts, wl.n_new, wl.K, sample, temp, seed)
         out = eng.alloc_step_outputs()
         for s in range(1, warmup + 1):
-            eng.step(out, step=s)
+            eng.step(out, sample, temp, seed, step=s)
         torch.cuda.synchronize()
         if ws > 1:
             torch.distributed.barrier()
         torch.cuda.synchronize()
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
         ph = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(timed_steps)]
-        n_emit = torch.zeros(timed_steps, dtype=torch.int32, device="cuda")
+        n_emit = torch.zeros((timed_steps, wl.batch), dtype=torch.int32, device="cuda")
         launches = 0
         ev[0].record(stream)
         for i in range(timed_steps):
             s = warmup + 1 + i
             if phase_events:
                 ph[i][0].record(stream)
-            eng.draft(out, False, 1.0, 0, s)
+            eng.draft(out, sample, temp, seed, s)
             launches += eng.launch_count()
             if phase_events:
                 ph[i][1].record(stream)
-            eng.verify(out, None, 1.0)
+            eng.verify(out, None, temp)
             launches += eng.launch_count()
             if phase_events:
                 ph[i][2].record(stream)
-            eng.accept_commit(out, False, 1.0, 0, s)
+            eng.accept_commit(out, sample, temp, seed, s)
             launches += eng.launch_count()
             if phase_events:
                 ph[i][3].record(stream)
-            n_emit[i:i + 1].copy_(out["n_emit"][:1])
+            n_emit[i].copy_(out["n_emit"])
         ev[1].record(stream)
         torch.cuda.synchronize()
         ms = ev[0].elapsed_time(ev[1])
@@ -330,30 +340,31 @@ def main():
     def e2e_run():
         h_prompt = torch.tensor([t for p in prompts for t in p], dtype=torch.int32).pin_memory()
         d_prompt = torch.empty_like(h_prompt, device="cuda")
-        h_out = torch.empty((wl.K + 1 + 1,), dtype=torch.int32).pin_memory()
+        B = wl.batch
+        h_out = torch.empty((B * (wl.K + 2),), dtype=torch.int32).pin_memory()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         d_prompt.copy_(h_prompt, non_blocking=True)
-        first = torch.empty(wl.batch, dtype=torch.int32, device="cuda")
-        lens_c = (pard.ctypes.c_int32 * wl.batch)(*lens)
+        first = torch.empty(B, dtype=torch.int32, device="cuda")
+        lens_c = (pard.ctypes.c_int32 * B)(*lens)
         pard._check(pard.lib().pard_prefill(eng.ctx, d_prompt.data_ptr(), pard.ctypes.cast(lens_c, pard.ctypes.c_void_p),
-                                            wl.batch, wl.n_new, wl.K, 0, 1.0, 0, first.data_ptr(),
+                                            B, wl.n_new, wl.K, int(sample), temp, seed, first.data_ptr(),
                                             stream.cuda_stream), "pard_prefill")
-        eng.batch, eng.K = wl.batch, wl.K
+        eng.batch, eng.K = B, wl.K
         out = eng.alloc_step_outputs()
-        gen = 1
+        gen = B  # the first token of every sequence
         steps = 0
-        while gen < wl.n_new:
+        while gen < B * wl.n_new and steps < 4 * wl.n_new:
             steps += 1
-            eng.step(out, step=steps)
-            h_out[: wl.K + 1].copy_(out["emitted"][0], non_blocking=True)
-            h_out[wl.K + 1:].copy_(out["n_emit"][:1], non_blocking=True)
+            eng.step(out, sample, temp, seed, step=steps)
+            h_out[: B * (wl.K + 1)].copy_(out["emitted"].reshape(-1), non_blocking=True)
+            h_out[B * (wl.K + 1):].copy_(out["n_emit"], non_blocking=True)
             torch.cuda.current_stream().synchronize()
-            gen += int(h_out[wl.K + 1])
+            gen += int(h_out[B * (wl.K + 1):].sum())
         dt = time.perf_counter() - t0
-        return gen / dt, steps, h_prompt.numel() * 4
+        return gen / dt, steps, h_prompt.numel() * 4, B * (wl.K + 2) * 4
 
-    e2e_tps, e2e_steps, prompt_bytes = e2e_run() if not args.no_e2e else (None, 1, 0)
+    e2e_tps, e2e_steps, prompt_bytes, d2h_bytes = e2e_run() if not args.no_e2e else (None, 1, 0, 0)
 
     # planted acceptance: the verify input is the target's own greedy
     # continuation with each candidate corrupted with probability 1 - alpha, so
@@ -403,7 +414,8 @@ def main():
                 "note": "verify input = the target's greedy continuation with each candidate corrupted "
                         "with probability 1 - alpha (seeded); draft still runs every step"}
 
-    planted = planted_run(0.90, 24) if not args.layers else None
+    headline = args.workload == "8b_greedy" and not args.layers
+    planted = planted_run(0.90, 24) if headline else None
 
     # autoregressive baseline on the same kernels: the target alone, one token
     # per verify + accept (K = 0), the decoding the paper's speedups are against
@@ -426,7 +438,7 @@ def main():
         return {"value": toks / (ms / 1e3), "unit": "tokens/s", "ms_per_token": ms / max(toks, 1), "steps": n_steps,
                 "note": "target alone, one token per step (pard_prefill K = 0: verify + accept, no draft)"}
 
-    ar = ar_run(30) if not args.layers else None
+    ar = ar_run(30) if headline else None
     if planted and ar:
         planted["speedup_vs_autoregressive"] = planted["value"] / ar["value"]
 
@@ -435,7 +447,8 @@ def main():
     ver_ms = statistics.median(phases["verify"])
     dr_ms = statistics.median(phases["draft"])
     acc_ms = statistics.median(phases["accept"])
-    ctx_mid = max(lens) + args.warmup + args.steps / 2.0  # mean context during the timed steps (a ~ 0)
+    # mean context during the timed steps, summed over the batch (a ~ 0 with random-init drafts)
+    ctx_mid = sum(lens) + wl.batch * (args.warmup + args.steps / 2.0)
     vb = verify_bytes(wl, ctx_mid)
     db = draft_bytes(wl, ctx_mid)
     ver_gbs = vb / (ver_ms / 1e3) / 1e9
@@ -455,7 +468,7 @@ def main():
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights and prompt ids)",
-        "config": {"workload": "8b_greedy: " + WORKLOAD_DESC, "parallelism": f"replicas{ws}",
+        "config": {"workload": (args.workload + ": " + WORKLOAD_DESCS[args.workload]), "parallelism": f"replicas{ws}",
                    "l2": "inputs larger than L2: 17.5 GB of weights stream from HBM every step",
                    "acceptance": "random-init draft: ~0 candidates accepted, ~1 token per step",
                    "forward_pass": "persistent" if fused_used else "per_phase"},
@@ -463,7 +476,9 @@ def main():
                      "kernel": ("verify pass: embedding kernel + one persistent fwd_kernel launch" if fused_used
                                 else "verify pass (all its launches; GEMM-dominated)"),
                      "achieved": ver_gbs, "peak": peak, "unit": "GB/s", "frac": ver_gbs / peak,
-                     "peak_kind": peak_kind, "traffic": None if args.layers else measured_verify_traffic(fused_used),
+                     "peak_kind": peak_kind,
+                     "traffic": (measured_verify_traffic(fused_used)
+                                 if args.workload == "8b_greedy" and not args.layers else None),
                      "traffic_source": "profiles/verify_pass_dram_traffic_8b.json (ncu DRAM bytes, 2-layer capture "
                                        "scaled to 32 layers; null if the kernels changed since)",
                      "bytes_per_launch": vb,
@@ -476,7 +491,7 @@ def main():
                        "tokens_per_s": tok_per_step_proj / (step_ms / 1e3),
                        "note": "acceptance rate from the paper (context); same measured step time"},
         "e2e": None if args.no_e2e else {"value": e2e_tps, "unit": "tokens/s", "h2d_bytes_per_step": prompt_bytes / max(e2e_steps, 1),
-                "d2h_bytes_per_step": 4 * (wl.K + 2),
+                "d2h_bytes_per_step": d2h_bytes,
                 "note": "full generation through the C ABI: pinned host prompt in, prefill, every step's tokens out"},
         "gpu_launches": launches,
         "clocks": clk,

@@ -172,6 +172,22 @@ def test_autoregressive_mode_k0_matches_the_oracle_forward():
     print("stats", stats)
 
 
+def test_batch16_ragged_full_width_two_layers():
+    """The batch-16 ragged configuration (8b_batch16: K = 6, ragged prompts)
+    at full width with two layers per model: 16 x 7 = 112 verify rows and 192
+    draft rows take the 64-token tiles, and attention covers 16 sequences of
+    different lengths.  Prompts are 16..64 tokens here (the configuration's
+    128..2048 keep the CPU oracle's prefill within seconds only at this size)."""
+    wl = S.WORKLOADS["8b_batch16"].replace(target=S.TARGET_8B.replace(n_layers=2),
+                                           draft=S.DRAFT_1B.replace(n_layers=2), prompt_len_range=(16, 64), n_new=12)
+    P = Pair(wl, prefill_chunk=64)
+    P.prefill()
+    for step in range(1, 4):
+        greedy_step(P, step)
+    assert P.eng.last_status() == 0
+    print("stats", P.stats)
+
+
 # ----------------------------------------------------------------------------
 # speculative sampling
 # ----------------------------------------------------------------------------
@@ -249,6 +265,44 @@ def test_sampling_end_to_end_tiny():
         slots, _ = P.oracle.commit([a_g], [em if len(em) == a_g + 1 else em + [0] * (a_g + 1 - len(em))])
         assert np.array_equal(out["kv_slots"][0].cpu().numpy()[: a_g + 1], slots[0][: a_g + 1])
         step += 1
+    assert checked > 0
+    assert P.eng.last_status() == 0
+
+
+def test_sampling_full_width_8b_two_layers():
+    """The sampling configuration (8b_sample: T = 1, K = 6) at full width with
+    two layers per model, 64-token prompt: logits within tolerance, accept
+    decisions equal wherever |u - p/q| > 1e-3, KV slots equal."""
+    wl = S.WORKLOADS["8b_sample"].replace(target=S.TARGET_8B.replace(n_layers=2),
+                                          draft=S.DRAFT_1B.replace(n_layers=2), prompt_len=64, n_new=16)
+    P = Pair(wl, prefill_chunk=64)
+    seed = 5
+    P.prefill(seed)
+    K = wl.K
+    checked = 0
+    for step in range(1, 4):
+        out = P.eng.alloc_step_outputs(want_logits=True)
+        P.eng.draft(out, True, 1.0, seed, step)
+        d_g = out["draft"].cpu().numpy()
+        z_g = out["draft_logits"].cpu().numpy()
+        d_o, z_o = P.oracle.draft(step, seed)
+        assert np.abs(z_g - z_o).max() <= LOGIT_TOL
+        P.eng.verify(out, None, 1.0)
+        y_g = out["logits"].cpu().numpy()
+        y_o = P.oracle.verify(d_g)
+        assert np.abs(y_g - y_o).max() <= LOGIT_TOL
+        P.eng.accept_commit(out, True, 1.0, seed, step)
+        a_g = int(out["accept_len"][0])
+        for i in range(min(a_g + 1, K)):
+            p = OP.softmax_t(y_o[0, i], 1.0)[d_g[0, i]]
+            q = OP.softmax_t(z_o[0, i], 1.0)[d_g[0, i]]
+            u = uniform01(raw_words(seed, STREAM_ACCEPT, step, 0, i, np.zeros(1, np.uint64)))[0]
+            if abs(u - p / q) > 1e-3:
+                assert (u * q < p) == (i < a_g), (step, i)
+                checked += 1
+        em = [int(x) for x in out["emitted"][0].cpu().numpy()[: a_g + 1]]
+        slots, _ = P.oracle.commit([a_g], [em if len(em) == a_g + 1 else em + [0] * (a_g + 1 - len(em))])
+        assert np.array_equal(out["kv_slots"][0].cpu().numpy()[: a_g + 1], slots[0][: a_g + 1])
     assert checked > 0
     assert P.eng.last_status() == 0
 
