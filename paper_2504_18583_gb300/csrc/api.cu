@@ -340,8 +340,8 @@ void run_gemm(pard_ctx* c, GemmArgs& a, int tt, cudaStream_t s) {
 }
 
 // Attention work decomposition of a pass: row blocks per sequence, groups
-// (sequence x kv head x row block) and key splits (<= 8, enough CTAs to cover
-// the GPU, at most one per 64-key chunk of the longest context).
+// (sequence x kv head x row block) and key splits (<= 16, about two CTAs per
+// SM, at most one per 32-key chunk of the longest context).
 struct AttnGeom {
   int row_blocks, groups, n_split;
 };

@@ -44,18 +44,6 @@ struct FwdCfg {
   static constexpr int kSmem = 1024 + kRing + kAttn + kPhase + kBar + kMisc + 4 * kEpiFloats + kSmall + 128;
 };
 
-__device__ __forceinline__ unsigned ld_relaxed_u32(const unsigned* p) {
-  unsigned v;
-  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
-  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-// with a preceding relaxed read that saw a released value: acquire
-__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
-// orders this thread's generic-proxy global accesses with its async-proxy (bulk copy) ones
-__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 __device__ __forceinline__ bool reached(unsigned v, unsigned target) { return (int)(v - target) >= 0; }
 
 // Phase p complete in every CTA, as seen by a relaxed read (no acquire yet:

@@ -14,8 +14,11 @@
 //    with TMA (128-byte swizzle) through a multi-stage mbarrier ring, warp 1
 //    issues tcgen05.mma into a TMEM accumulator, warps 2-5 drain TMEM;
 //  * the flattened (tile, K-chunk) index space is split evenly over the
-//    CTAs; a tile shared by several CTAs is finished by the last one to
-//    arrive, which sums the partials in CTA order (deterministic);
+//    CTAs; a tile shared by several CTAs is finished by the first of them,
+//    for which it is the last segment: the others store their partials and
+//    signal with one release increment each, the finisher pulls all partials
+//    into its idle stage ring with bulk copies and sums them in CTA order
+//    (deterministic);
 //  * epilogues are fused: RMS row scaling, RoPE + paged KV write (QKV),
 //    residual add + next norm's gain and sum of squares (O / down),
 //    SiLU(gate) * up (gate/up pairs), logits + per-tile max / argmax /
@@ -39,10 +42,12 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
   uint64_t* accf = empty + C::kStages;
   uint64_t* acce = accf + 2;
   uint64_t* drain = acce + 2;
-  uint32_t* misc = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* fx = drain + 1;  // split-K finish: partials pulled into the ring
+  uint32_t* misc = reinterpret_cast<uint32_t*>(drain + 2);
   uint32_t* tmem_slot = misc;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
   int* bcast = reinterpret_cast<int*>(misc + 2);
+  volatile int* fx_armed = reinterpret_cast<volatile int*>(misc + 3);
   float* scratch = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(misc) + C::kMiscBytes);
   const EpiSmem S = carve_epi<TT>(scratch);
 
@@ -56,7 +61,9 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
     for (int s = 0; s < C::kStages; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     for (int b = 0; b < 2; ++b) { mbar_init(&accf[b], 1); mbar_init(&acce[b], 128); }
     mbar_init(drain, 1);
+    mbar_init(fx, 1);
     *abort_flag = 0;
+    *fx_armed = 0;
     fence_barrier_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
@@ -206,6 +213,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       M = a.m_cap;
     }
     int seg_i = 0;
+    int rs_tok = -1;  // token tile whose RMS row scale S.rs holds
     for (long u = u0; u < u1;) {
       const long t = u / a.kc;
       const long ub = u, ue = (t + 1) * a.kc < u1 ? (t + 1) * a.kc : u1;
@@ -213,7 +221,14 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       const int ab = seg_i % C::kNumAcc;
       const int w_tile = (int)(t / a.tok_tiles), tok_tile = (int)(t % a.tok_tiles);
       const int tok_base = tok_tile * TT;
-      if (a.ssq_in) epi_row_scale<TT>(a, tok_base, et, M, S);
+      if (a.ssq_in && tok_base != rs_tok) {
+        epi_row_scale<TT>(a, tok_base, et, M, S);
+        rs_tok = tok_base;
+      }
+      // result-independent loads of a segment this CTA finishes (it starts
+      // the tile), issued while the MMAs run
+      EpiPre pre0 = {};
+      if (ub == t * a.kc) pre0 = epi_pre(a, w_tile, tok_base, et, M);
       if (!mbar_wait(&accf[ab], (uint32_t)((seg_i / C::kNumAcc) & 1), abort_flag)) {
         if (et == 0) set_status(a.status, ST_TIMEOUT_EPI);
         *abort_flag = 1;
@@ -222,7 +237,10 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       tc_fence_after();
       epi_bar();
       const uint32_t tbase = tmem + ab * C::kAccCols + ((uint32_t)(q * 32) << 16);
-      epi_segment<TT>(a, t, ub, ue, u0, U, G, c, tbase, w_tile, tok_base, fr, et, M, S, bcast);
+      if (!epi_segment_owned<TT>(a, t, ub, ue, u0, U, G, c, tbase, w_tile, tok_base, fr, et, M, S, pre0,
+                                 reinterpret_cast<float*>(sA), (uint32_t)(C::kStages * C::kStageBytes), fx,
+                                 fx_armed, abort_flag, bcast))
+        break;
       tc_fence_before();
       mbar_arrive(&acce[ab]);
       epi_bar();
@@ -241,6 +259,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       umma_commit(drain);
       mbar_drain(drain, 0);
     }
+    if (threadIdx.x == 64 && *fx_armed) mbar_drain(fx, 0);
     __syncthreads();
   }
   if (warp == 1) {

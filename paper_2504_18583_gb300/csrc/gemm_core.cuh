@@ -22,7 +22,7 @@ struct GemmCfg {
                                    : kNumAcc * kAccCols <= 128 ? 128 : 256;
   static constexpr int kChunks = TT / kEpiTok;
   // scratch after the stage ring
-  static constexpr int kBarBytes = 8 * (2 * kStages + 5);  // full, empty, accf x2, acce x2, drain
+  static constexpr int kBarBytes = 8 * (2 * kStages + 6);  // full, empty, accf x2, acce x2, drain, fix-up
   static constexpr int kMiscBytes = 64;
   static constexpr int kScratchFloats = TT + 4 * 64 + 16 + kEpiTok * kTileN + 3 * kEpiTok;
   static constexpr int kSmem = 1024 + kStages * kStageBytes + kBarBytes + kMiscBytes + 4 * kScratchFloats;
@@ -497,6 +497,138 @@ __device__ void epi_segment(const GemmArgs& a, long t, long ub, long ue, long u0
       if (et == 0) a.counters[t] = 0;
     }
   }
+}
+
+// Bounded wait until *p >= target, with acquire semantics on success.
+__device__ __forceinline__ bool wait_count(const int* p, int target, volatile int* abort) {
+  if (ld_acquire_s32(p) >= target) return true;
+  const unsigned long long t0 = globaltimer();
+  while (true) {
+    if (ld_acquire_s32(p) >= target) return true;
+    if (*abort) return false;
+    if (globaltimer() - t0 > kWaitLimitNs) return false;
+  }
+}
+
+// Split-K with a designated finisher (per-phase kernel).  The first CTA of a
+// tile in CTA order, cf, finishes it.  Its share of the tile is the last
+// segment of its range (the tile starts inside the range and runs past its
+// end), so when its epilogue gets there every MMA of the CTA has completed and
+// the stage ring is idle.  The other contributors store their partial, make
+// one release increment of the tile's counter and move on without a round
+// trip.  cf waits for the cl - cf increments, pulls every partial into the
+// ring with one bulk copy each (a single round trip for the whole tile) and
+// sums in CTA order, itself first: the same order, so the same sums, as the
+// last-arriver scheme of epi_segment.  pre0: epi_pre of the segment's first
+// chunk, taken by the caller before the accumulator was ready; only read for
+// a whole tile or by cf.  ring/ring_bytes: the stage ring; fx: an mbarrier
+// used once per launch; fx_armed: set while its copies are in flight.
+template <int TT>
+__device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, long u0, long U, long G, long c,
+                                  uint32_t tbase, int w_tile, int tok_base, int fr, int et, int M, const EpiSmem& S,
+                                  const EpiPre& pre0, float* ring, uint32_t ring_bytes, uint64_t* fx,
+                                  volatile int* fx_armed, volatile int* abort_flag, int* bcast) {
+  using C = GemmCfg<TT>;
+  constexpr int kTileF = kTileN * TT;  // floats of one partial tile
+  if (ub == t * a.kc && ue == (t + 1) * a.kc) {
+#pragma unroll 1
+    for (int ch = 0; ch < C::kChunks; ++ch) {
+      uint32_t r[32];
+      tmem_ld32(tbase + ch * 32, r);
+      float v[kEpiTok];
+#pragma unroll
+      for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
+      epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S,
+                ch == 0 ? pre0 : epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M));
+    }
+    return true;
+  }
+  const long cf = owner_of(t * a.kc, U, G), cl = owner_of((t + 1) * a.kc - 1, U, G);
+  if (c != cf) {
+    const int slot = (ub == u0) ? 0 : 1;
+    float* mine = a.partials + ((size_t)c * 2 + slot) * kTileF;
+#pragma unroll 1
+    for (int ch = 0; ch < C::kChunks; ++ch) {
+      uint32_t r[32];
+      tmem_ld32(tbase + ch * 32, r);
+      float4* dst = reinterpret_cast<float4*>(mine + ((size_t)ch * kTileN + fr) * kEpiTok);
+#pragma unroll
+      for (int j4 = 0; j4 < 4; ++j4)
+        dst[j4] = make_float4(__uint_as_float(r[8 * j4 + 0]) + __uint_as_float(r[8 * j4 + 1]),
+                              __uint_as_float(r[8 * j4 + 2]) + __uint_as_float(r[8 * j4 + 3]),
+                              __uint_as_float(r[8 * j4 + 4]) + __uint_as_float(r[8 * j4 + 5]),
+                              __uint_as_float(r[8 * j4 + 6]) + __uint_as_float(r[8 * j4 + 7]));
+    }
+    // the barrier orders every thread's partial before the one release
+    // increment (cumulative)
+    epi_bar();
+    if (et == 0) red_release_add(reinterpret_cast<unsigned*>(&a.counters[t]), 1u);
+    return true;
+  }
+  const int n_other = (int)(cl - cf);
+  const bool staged = (uint32_t)n_other * kTileF * 4 <= ring_bytes;
+  if (et == 0) {
+    const bool ok = wait_count(&a.counters[t], n_other, abort_flag);
+    if (!ok) set_status(a.status, ST_TIMEOUT_EPI);
+    if (ok && staged) {
+      // the partials were written through the generic proxy; the copies read
+      // them through the async proxy
+      fence_proxy_async();
+      *fx_armed = 1;
+      mbar_arrive_expect_tx(fx, (uint32_t)n_other * kTileF * 4);
+      for (int k = 0; k < n_other; ++k) {
+        const long cc = cf + 1 + k;
+        const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
+        bulk_load(ring + (size_t)k * kTileF, a.partials + ((size_t)cc * 2 + sl) * kTileF, kTileF * 4, fx);
+      }
+    }
+    bcast[0] = ok ? 1 : 0;
+  }
+  epi_bar();
+  if (!bcast[0]) {
+    *abort_flag = 1;
+    return false;
+  }
+  const bool late = staged && !mbar_wait(fx, 0, abort_flag);
+  if (epi_bar_any(late)) {
+    if (et == 0) set_status(a.status, ST_TIMEOUT_EPI);
+    *abort_flag = 1;
+    return false;
+  }
+#pragma unroll 1
+  for (int ch = 0; ch < C::kChunks; ++ch) {
+    uint32_t r[32];
+    tmem_ld32(tbase + ch * 32, r);
+    float v[kEpiTok];
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
+    const size_t off = ((size_t)ch * kTileN + fr) * kEpiTok;
+    for (int k = 0; k < n_other; ++k) {
+      float4 pv[4];
+      if (staged) {
+        const float4* p = reinterpret_cast<const float4*>(ring + (size_t)k * kTileF + off);
+#pragma unroll
+        for (int j4 = 0; j4 < 4; ++j4) pv[j4] = p[j4];
+      } else {
+        const long cc = cf + 1 + k;
+        const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
+        const float4* p = reinterpret_cast<const float4*>(a.partials + ((size_t)cc * 2 + sl) * kTileF + off);
+#pragma unroll
+        for (int j4 = 0; j4 < 4; ++j4) pv[j4] = __ldcg(p + j4);
+      }
+#pragma unroll
+      for (int j4 = 0; j4 < 4; ++j4) {
+        v[4 * j4 + 0] += pv[j4].x;
+        v[4 * j4 + 1] += pv[j4].y;
+        v[4 * j4 + 2] += pv[j4].z;
+        v[4 * j4 + 3] += pv[j4].w;
+      }
+    }
+    epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S,
+              ch == 0 ? pre0 : epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M));
+  }
+  if (et == 0) a.counters[t] = 0;
+  return true;
 }
 
 // RMS row scale for the token tile starting at tok_base: all partial sums of
