@@ -27,16 +27,18 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_pos[kMaxQV];
 
-  pdl_wait();
   const uint32_t rank = cluster_rank(), NS = cluster_size();
   const int group_idx = blockIdx.x / NS;
   const int rb = group_idx % a.row_blocks;
   const int kvh = (group_idx / a.row_blocks) % a.hkv;
   const int b = group_idx / (a.row_blocks * a.hkv);
-  // with a fixed row count per sequence the row range needs no load
-  const int M = a.rows_per_seq > 0 ? a.batch * a.rows_per_seq : *a.m_dev;
+  // Row plan, positions, page tables and the keys and values of earlier
+  // passes are written before the previous kernel (the QKV projection), which
+  // had itself waited for them before it let this grid start: the unit reads
+  // them before waiting, and Q after.
+  const int M = a.rows_per_seq > 0 ? a.batch * a.rows_per_seq : __ldcg(a.m_dev);
   const AttnRows R = attn_unit<HD, GROUP, kAttnBufs>(a, b, kvh, rb, (int)rank, (int)NS, M, smem, s_pos,
-                                                     threadIdx.x, [] { __syncthreads(); });
+                                                     threadIdx.x, [] { __syncthreads(); }, [] { pdl_wait(); });
   const int row0 = R.row0, nqv = R.nrows * GROUP;
   // the next kernel may start streaming its weights once the key/value reads
   // are done: earlier, its bulk loads would queue ahead of them

@@ -154,12 +154,16 @@ struct AttnRows {
 // other warps'), and its row positions in s_pos[64].  bar() synchronises the
 // 128 threads.
 //
-// Latency structure: one round of loads brings the row positions, Q and the
-// sequence's page table row together; then NBUF - 1 chunks of K/V stay in
-// flight while the warps compute on the oldest.
-template <int HD, int GROUP, int NBUF, typename Bar>
+// Latency structure: a first round of loads brings the row positions, the
+// sequence's first position in this pass and its page table row, none of
+// which the producer of Q writes; the chunks wholly below that first
+// position (keys and values of earlier passes) are requested next, and only
+// then does the unit call wait_q() (the standalone kernel's wait on the
+// previous kernel).  A second round brings Q, the remaining chunks follow, and
+// NBUF - 1 chunks stay in flight while the warps compute on the oldest.
+template <int HD, int GROUP, int NBUF, typename Bar, typename WaitQ>
 __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp, int ns, int M, uint8_t* smem,
-                              int* s_pos, int tid, Bar bar) {
+                              int* s_pos, int tid, Bar bar, WaitQ wait_q) {
   static_assert(NBUF >= 2 && NBUF <= 4, "chunk ring of 2 to 4 buffers");
   using C = AttnCfg<HD, NBUF>;
   constexpr int RB = kMaxQV / GROUP;  // rows per block
@@ -170,8 +174,9 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
   const int g = lane >> 2, c4 = lane & 3;
 
   AttnRows R{0, 0};
+  int s0 = 0;
   if (b < a.batch) {
-    const int s0 = a.rows_per_seq > 0 ? b * a.rows_per_seq : a.seq_row0[b];
+    s0 = a.rows_per_seq > 0 ? b * a.rows_per_seq : a.seq_row0[b];
     const int s1 = a.rows_per_seq > 0 ? s0 + a.rows_per_seq : a.seq_row0[b + 1];
     R.row0 = s0 + rb * RB;
     const int row_end = min(min(s1, R.row0 + RB), M);
@@ -184,14 +189,39 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
   int* spg = reinterpret_cast<int*>(smem + C::kPageOff);
   const bool cached = a.pt_ld <= kAttnPageCache;
 
-  // ---- one round of loads: row positions, page table row, Q ----
-  const int pos_v = tid < nrows ? a.row_pos[row0 + tid] : -1;
+  // ---- round 1: row positions, the sequence's first position, page table row ----
+  const int pos_v = tid < nrows ? __ldcg(a.row_pos + row0 + tid) : -1;
+  const int first_v = (tid == 0 && nrows > 0) ? __ldcg(a.row_pos + s0) : 0;
   int pg_v[kAttnPageCache / kAttnThreads];
 #pragma unroll
   for (int k = 0; k < kAttnPageCache / kAttnThreads; ++k) {
     const int i = tid + k * kAttnThreads;
-    pg_v[k] = (cached && i < a.pt_ld) ? pt[i] : -1;
+    pg_v[k] = (cached && i < a.pt_ld) ? __ldcg(pt + i) : -1;
   }
+  if (tid < kMaxQV) s_pos[tid] = pos_v;
+  if (tid == 0) spg[kAttnPageCache] = first_v;
+#pragma unroll
+  for (int k = 0; k < kAttnPageCache / kAttnThreads; ++k) spg[tid + k * kAttnThreads] = pg_v[k];
+  bar();
+  int maxpos = -1;
+  for (int r = 0; r < nrows; ++r) maxpos = max(maxpos, s_pos[r]);
+  const int first_new = spg[kAttnPageCache];  // keys from here on are written by this pass
+  const int n_chunks = maxpos >= 0 ? maxpos / kKeyChunk + 1 : 0;
+  const int c0 = (int)((long)sp * n_chunks / ns), c1 = (int)((long)(sp + 1) * n_chunks / ns);
+  const int n = c1 - c0;
+  const int* pgs = cached ? spg : nullptr;
+
+  // ---- chunks of earlier passes: in flight before Q is available ----
+  auto kbuf = [&](int t) { return smem + (t % NBUF) * 2 * C::kTileBytes; };
+  int issued = 0;
+  for (; issued < n && issued < NBUF - 1 && (c0 + issued + 1) * kKeyChunk <= first_new; ++issued) {
+    uint8_t* k = kbuf(issued);
+    load_chunk<HD, NBUF>(a, pt, pgs, kvh, c0 + issued, maxpos, k, k + C::kTileBytes, tid);
+    cp_async_commit();
+  }
+  wait_q();
+
+  // ---- round 2: Q ----
   // q is rewritten by every layer, by other CTAs of a persistent grid: L2 loads
   constexpr int kQIter = kMaxQV * (HD / 4) / kAttnThreads;  // 8 or 16 float4 per thread
   constexpr int kQGroup = kQIter < 8 ? kQIter : 8;
@@ -214,22 +244,11 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
           make_uint2(pack_h2(v[u].x, v[u].y), pack_h2(v[u].z, v[u].w));
     }
   }
-  if (tid < kMaxQV) s_pos[tid] = pos_v;
-#pragma unroll
-  for (int k = 0; k < kAttnPageCache / kAttnThreads; ++k) spg[tid + k * kAttnThreads] = pg_v[k];
   bar();
-  int maxpos = -1;
-  for (int r = 0; r < nrows; ++r) maxpos = max(maxpos, s_pos[r]);
-  const int n_chunks = maxpos >= 0 ? maxpos / kKeyChunk + 1 : 0;
-  const int c0 = (int)((long)sp * n_chunks / ns), c1 = (int)((long)(sp + 1) * n_chunks / ns);
-  const int n = c1 - c0;
-  const int* pgs = cached ? spg : nullptr;
   const int qa = warp * 16 + g, qb = qa + 8;
   const int posa = qa < nqv ? s_pos[qa / GROUP] : -1, posb = qb < nqv ? s_pos[qb / GROUP] : -1;
 
   // ---- K/V chunk ring: NBUF - 1 chunks in flight ----
-  auto kbuf = [&](int t) { return smem + (t % NBUF) * 2 * C::kTileBytes; };
-  int issued = 0;
   for (; issued < n && issued < NBUF - 1; ++issued) {
     uint8_t* k = kbuf(issued);
     load_chunk<HD, NBUF>(a, pt, pgs, kvh, c0 + issued, maxpos, k, k + C::kTileBytes, tid);

@@ -401,7 +401,7 @@ __global__ void __launch_bounds__(192, 1) fwd_kernel(const __grid_constant__ Fwd
           const int kvh = (gidx / at.row_blocks) % at.hkv;
           const int b = gidx / (at.row_blocks * at.hkv);
           const AttnRows R = attn_unit<HD, GROUP, F::kAttnBufs>(at, b, kvh, rb, sp, ns, M, sAttn, s_pos, et,
-                                                                [] { epi_bar(); });
+                                                                [] { epi_bar(); }, [] {});
           const int row0 = R.row0, nqv = R.nrows * GROUP;
           epi_bar();  // every warp's partial is in shared memory
           const float* part = reinterpret_cast<const float*>(sAttn);
