@@ -207,7 +207,11 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
   for (int r = 0; r < nrows; ++r) maxpos = max(maxpos, s_pos[r]);
   const int first_new = spg[kAttnPageCache];  // keys from here on are written by this pass
   const int n_chunks = maxpos >= 0 ? maxpos / kKeyChunk + 1 : 0;
-  const int c0 = (int)((long)sp * n_chunks / ns), c1 = (int)((long)(sp + 1) * n_chunks / ns);
+  // contiguous chunk ranges; the remainder goes to the first splits, so the
+  // last one, which holds this pass's own keys (read only after wait_q),
+  // has the fewest
+  const int base = n_chunks / ns, rem = n_chunks % ns;
+  const int c0 = sp * base + min(sp, rem), c1 = c0 + base + (sp < rem ? 1 : 0);
   const int n = c1 - c0;
   const int* pgs = cached ? spg : nullptr;
 
