@@ -24,10 +24,22 @@ constexpr int kAttnBufs = 4;  // K/V chunk ring of the standalone kernel (3 chun
 
 template <int HD, int GROUP>
 __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constant__ AttnArgs a) {
+  using C = AttnCfg<HD, kAttnBufs>;
+  constexpr int LD = C::kPartLd;
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_pos[kMaxQV];
+  __shared__ __align__(8) uint64_t s_recv;  // push combine: this CTA's incoming partials
+  __shared__ int s_flag;                    // never raised: the wait below has no other role to abort it
 
   const uint32_t rank = cluster_rank(), NS = cluster_size();
+  if (threadIdx.x == 0) {
+    mbar_init(&s_recv, 1);
+    s_flag = 0;
+    fence_barrier_init();
+  }
+  // first cluster barrier: every CTA's s_recv is initialised (waited on
+  // before any partial is pushed)
+  cluster_arrive_relaxed();
   const int group_idx = blockIdx.x / NS;
   const int rb = group_idx % a.row_blocks;
   const int kvh = (group_idx / a.row_blocks) % a.hkv;
@@ -44,11 +56,79 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
   // are done: earlier, its bulk loads would queue ahead of them
   pdl_trigger();
   float* part = reinterpret_cast<float*>(smem);
+
+  // Push combine: CTA o finishes query vectors [o cnt, (o + 1) cnt).  Every
+  // CTA copies those rows of its partial into CTA o's shared memory with one
+  // bulk copy, counted on o's s_recv, so a CTA waits only for its own inputs
+  // and reads them locally.  The receive area is the part of the K/V ring that
+  // no CTA of the cluster uses (each walks at most max_n chunks) above this
+  // CTA's own partial; when it does not fit, the cluster pulls instead.
+  const int cnt = (nqv + (int)NS - 1) / (int)NS;
+  const int max_n = (R.n_chunks + (int)NS - 1) / (int)NS;
+  // the partial rows written: every active warp writes all 16 of its rows
+  const uint32_t part_bytes = (uint32_t)((nqv + 15) / 16 * 16) * LD * 4;
+  const uint32_t ring_used = (uint32_t)max_n * 2 * C::kTileBytes;
+  const uint32_t recv_off = ((ring_used > part_bytes ? ring_used : part_bytes) + 127) & ~127u;
+  const uint32_t recv_bytes = NS * (uint32_t)cnt * LD * 4;
+  const bool push = NS > 1 && recv_off + recv_bytes <= (uint32_t)C::kKV;
+  // every thread's partial writes, ordered before the async-proxy reads of
+  // the bulk copies below, and every warp's partial in shared memory
+  fence_proxy_async_smem();
+  __syncthreads();
+  cluster_wait();  // first barrier
+  if (push) {
+    float* recv = reinterpret_cast<float*>(smem + recv_off);  // [NS][cnt][LD]
+    const int my0 = (int)rank * cnt;
+    const int my_n = max(0, min(nqv, my0 + cnt) - my0);
+    if (threadIdx.x == 0 && my_n > 0) mbar_arrive_expect_tx(&s_recv, NS * (uint32_t)my_n * LD * 4);
+    if (threadIdx.x < NS) {
+      const uint32_t o = threadIdx.x;
+      const int r0 = (int)o * cnt, rn = max(0, min(nqv, r0 + cnt) - r0);
+      if (rn > 0) {
+        bulk_copy_to_peer(mapa_shared(recv + (size_t)rank * cnt * LD, o), part + (size_t)r0 * LD,
+                          (uint32_t)rn * LD * 4, mapa_shared(&s_recv, o));
+        bulk_commit();
+        bulk_wait_read_all();
+      }
+    }
+    // second barrier, arrive: this CTA's pushes are issued and their sources read
+    cluster_arrive();
+    bool ok = my_n == 0 || mbar_wait(&s_recv, 0, &s_flag);
+    if (!ok && threadIdx.x == 0) set_status(a.status, ST_TIMEOUT_EPI);
+    ok = __syncthreads_and(ok);
+    if (ok) {
+      for (int i = threadIdx.x; i < my_n * (HD / 4); i += kAttnThreads) {
+        const int r = i / (HD / 4), d4 = i % (HD / 4);
+        float mx = -INFINITY;
+        for (int sr = 0; sr < (int)NS; ++sr) mx = fmaxf(mx, recv[((size_t)sr * cnt + r) * LD + HD]);
+        float L = 0.f;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int sr = 0; sr < (int)NS; ++sr) {
+          const float* src = recv + ((size_t)sr * cnt + r) * LD;
+          const float m = src[HD];
+          const float w = m == -INFINITY ? 0.f : expf(m - mx);
+          L += src[HD + 1] * w;
+          const float4 v = *reinterpret_cast<const float4*>(src + 4 * d4);
+          acc.x += v.x * w;
+          acc.y += v.y * w;
+          acc.z += v.z * w;
+          acc.w += v.w * w;
+        }
+        const float inv = 1.0f / L;
+        const int qv = my0 + r;
+        store_pair4(a.x_out, row0 + qv / GROUP, (kvh * GROUP + qv % GROUP) * HD + 4 * d4, a.x_rows,
+                    make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv));
+      }
+    }
+    // second barrier, wait: no peer copies into this CTA any more
+    cluster_wait();
+    return;
+  }
   cluster_sync();
-  // combine in rank order; CTA `rank` finishes query vectors rank, rank+NS, ...
-  // Each thread takes one output pair (qv, d..d+1) at a time and requests
-  // every rank's (max, sum) and partial values before using any, so a round of
-  // work is one distributed-shared-memory round trip.
+  // Pull combine, in rank order; CTA `rank` finishes query vectors rank,
+  // rank+NS, ...  Each thread takes one output pair (qv, d..d+1) at a time
+  // and requests every rank's (max, sum) and partial values before using any,
+  // so a round of work is one distributed-shared-memory round trip.
   const int my_qv = nqv > (int)rank ? (nqv - (int)rank + (int)NS - 1) / (int)NS : 0;
   const int n_items = my_qv * (HD / 2);
   for (int i = threadIdx.x; i < n_items; i += kAttnThreads) {
@@ -57,8 +137,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
 #pragma unroll
     for (int r = 0; r < kMaxCluster; ++r) {
       const bool live = r < (int)NS;
-      ml[r] = live ? ld_dsmem2(part + qv * (HD + 2) + HD, (uint32_t)r) : make_float2(-INFINITY, 0.f);
-      pv[r] = live ? ld_dsmem2(part + qv * (HD + 2) + d, (uint32_t)r) : make_float2(0.f, 0.f);
+      ml[r] = live ? ld_dsmem2(part + qv * LD + HD, (uint32_t)r) : make_float2(-INFINITY, 0.f);
+      pv[r] = live ? ld_dsmem2(part + qv * LD + d, (uint32_t)r) : make_float2(0.f, 0.f);
     }
     float mx = -INFINITY;
 #pragma unroll

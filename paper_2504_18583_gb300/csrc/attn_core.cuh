@@ -28,7 +28,8 @@ struct AttnCfg {
   static constexpr int kKV = NBUF * 2 * kTileBytes;         // K and V chunk ring
   static constexpr int kQBytes = kMaxQV * kRowBytes;        // Q rows
   static constexpr int kQOff = kKV;
-  static constexpr int kPart = kMaxQV * (HD + 2) * 4;       // partial (o, m, l) per CTA
+  static constexpr int kPartLd = HD + 4;                     // partial row: o[HD], m, l, 2 pad (16-byte rows)
+  static constexpr int kPart = kMaxQV * kPartLd * 4;        // partial (o, m, l) per CTA
   static constexpr int kPageOff = (kKV + kQBytes) > kPart ? (kKV + kQBytes) : kPart;
   static constexpr int kSmem = kPageOff + kAttnPageCache * 4 + 256;
 };
@@ -85,6 +86,50 @@ __device__ __forceinline__ float2 ld_dsmem2(const float* local, uint32_t rank) {
   asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(remote) : "memory");
   return v;
 }
+
+// Four consecutive columns (col % 4 == 0) of activation row m as bf16 hi/lo
+// pairs in the packed layout: 8 contiguous bytes in each of rows 2m and 2m+1.
+__device__ __forceinline__ void store_pair4(__nv_bfloat16* x, int m, int col, int x_rows, float4 v) {
+  __nv_bfloat16 h[4], l[4];
+  split_bf16(v.x, h[0], l[0]);
+  split_bf16(v.y, h[1], l[1]);
+  split_bf16(v.z, h[2], l[2]);
+  split_bf16(v.w, h[3], l[3]);
+  uint2 hv, lv;
+  hv.x = (uint32_t)__bfloat16_as_ushort(h[0]) | ((uint32_t)__bfloat16_as_ushort(h[1]) << 16);
+  hv.y = (uint32_t)__bfloat16_as_ushort(h[2]) | ((uint32_t)__bfloat16_as_ushort(h[3]) << 16);
+  lv.x = (uint32_t)__bfloat16_as_ushort(l[0]) | ((uint32_t)__bfloat16_as_ushort(l[1]) << 16);
+  lv.y = (uint32_t)__bfloat16_as_ushort(l[2]) | ((uint32_t)__bfloat16_as_ushort(l[3]) << 16);
+  *reinterpret_cast<uint2*>(x + xpk(2 * m, col, x_rows)) = hv;
+  *reinterpret_cast<uint2*>(x + xpk(2 * m + 1, col, x_rows)) = lv;
+}
+
+// ---- cluster barrier halves, distributed shared memory bulk copies --------
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
+// shared::cluster address of the same offset in CTA `rank`'s shared memory
+__device__ __forceinline__ uint32_t mapa_shared(const void* local, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(local)), "r"(rank));
+  return r;
+}
+// bytes (multiple of 16, both ends 16-byte aligned) of this CTA's shared
+// memory into a peer's, completion counted on the peer's mbarrier
+__device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst_cluster, const void* src, uint32_t bytes,
+                                                  uint32_t mbar_cluster) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst_cluster),
+      "r"(smem_u32(src)), "r"(bytes), "r"(mbar_cluster)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// this thread's bulk copies have finished reading their sources
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// orders this thread's generic-proxy shared memory writes before its async-proxy reads
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 // K and V rows of one 32-key chunk into shared memory; positions past maxpos
 // (masked anyway) and bad pages become zeros.  spg: the sequence's page table
@@ -143,13 +188,14 @@ __device__ __forceinline__ void cp_async_wait_upto(int n) {
 
 struct AttnRows {
   int row0, nrows;
+  int n_chunks;  // 32-key chunks of the unit's key range (all splits)
 };
 
 // One attention work unit of 4 warps (tid 0..127, warp = tid / 32): sequence
 // b, kv head kvh, row block rb (rows row0 .. row0 + nrows - 1 of the pass,
 // query vectors qv = r * GROUP + head), key split sp of ns over the 32-key
 // chunks up to the block's last position.  Leaves the unnormalised output and
-// the softmax (max, sum) of each query vector in smem as [64][HD + 2] floats
+// the softmax (max, sum) of each query vector in smem as [64][kPartLd] floats
 // (each warp its own query vectors; the caller synchronises before reading
 // other warps'), and its row positions in s_pos[64].  bar() synchronises the
 // 128 threads.
@@ -173,7 +219,7 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
   const int warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, c4 = lane & 3;
 
-  AttnRows R{0, 0};
+  AttnRows R{0, 0, 0};
   int s0 = 0;
   if (b < a.batch) {
     s0 = a.rows_per_seq > 0 ? b * a.rows_per_seq : a.seq_row0[b];
@@ -207,6 +253,7 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
   for (int r = 0; r < nrows; ++r) maxpos = max(maxpos, s_pos[r]);
   const int first_new = spg[kAttnPageCache];  // keys from here on are written by this pass
   const int n_chunks = maxpos >= 0 ? maxpos / kKeyChunk + 1 : 0;
+  R.n_chunks = n_chunks;
   // contiguous chunk ranges; the remainder goes to the first splits, so the
   // last one, which holds this pass's own keys (read only after wait_q),
   // has the fewest
@@ -369,16 +416,16 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
       const int d = nt * 8 + 2 * c4;
-      part[qa * (HD + 2) + d] = o[nt][0];
-      part[qa * (HD + 2) + d + 1] = o[nt][1];
-      part[qb * (HD + 2) + d] = o[nt][2];
-      part[qb * (HD + 2) + d + 1] = o[nt][3];
+      part[qa * C::kPartLd + d] = o[nt][0];
+      part[qa * C::kPartLd + d + 1] = o[nt][1];
+      part[qb * C::kPartLd + d] = o[nt][2];
+      part[qb * C::kPartLd + d + 1] = o[nt][3];
     }
     if (c4 == 0) {
-      part[qa * (HD + 2) + HD] = ma;
-      part[qa * (HD + 2) + HD + 1] = la;
-      part[qb * (HD + 2) + HD] = mb;
-      part[qb * (HD + 2) + HD + 1] = lb;
+      part[qa * C::kPartLd + HD] = ma;
+      part[qa * C::kPartLd + HD + 1] = la;
+      part[qb * C::kPartLd + HD] = mb;
+      part[qb * C::kPartLd + HD + 1] = lb;
     }
   }
   return R;

@@ -156,23 +156,6 @@ __device__ __forceinline__ void prefetch_next(const FwdArgs& f, long c, long G, 
   ++q.u;
 }
 
-// Four consecutive columns (col % 4 == 0) of activation row m as bf16 hi/lo
-// pairs in the packed layout: 8 contiguous bytes in each of rows 2m and 2m+1.
-__device__ __forceinline__ void store_pair4(__nv_bfloat16* x, int m, int col, int x_rows, float4 v) {
-  __nv_bfloat16 h[4], l[4];
-  split_bf16(v.x, h[0], l[0]);
-  split_bf16(v.y, h[1], l[1]);
-  split_bf16(v.z, h[2], l[2]);
-  split_bf16(v.w, h[3], l[3]);
-  uint2 hv, lv;
-  hv.x = (uint32_t)__bfloat16_as_ushort(h[0]) | ((uint32_t)__bfloat16_as_ushort(h[1]) << 16);
-  hv.y = (uint32_t)__bfloat16_as_ushort(h[2]) | ((uint32_t)__bfloat16_as_ushort(h[3]) << 16);
-  lv.x = (uint32_t)__bfloat16_as_ushort(l[0]) | ((uint32_t)__bfloat16_as_ushort(l[1]) << 16);
-  lv.y = (uint32_t)__bfloat16_as_ushort(l[2]) | ((uint32_t)__bfloat16_as_ushort(l[3]) << 16);
-  *reinterpret_cast<uint2*>(x + xpk(2 * m, col, x_rows)) = hv;
-  *reinterpret_cast<uint2*>(x + xpk(2 * m + 1, col, x_rows)) = lv;
-}
-
 template <int HD, int GROUP>
 __global__ void __launch_bounds__(192, 1) fwd_kernel(const __grid_constant__ FwdArgs f) {
   constexpr int TT = kFwdTT, S = kFwdStages;
@@ -408,7 +391,7 @@ __global__ void __launch_bounds__(192, 1) fwd_kernel(const __grid_constant__ Fwd
           if (ns == 1) {
             for (int i = et; i < nqv * (HD / 4); i += 128) {
               const int qv = i / (HD / 4), d4 = i % (HD / 4);
-              const float* src = part + qv * (HD + 2);
+              const float* src = part + qv * AttnCfg<HD, F::kAttnBufs>::kPartLd;
               const float inv = 1.0f / src[HD + 1];
               const float4 v = make_float4(src[4 * d4] * inv, src[4 * d4 + 1] * inv, src[4 * d4 + 2] * inv,
                                            src[4 * d4 + 3] * inv);
@@ -423,12 +406,13 @@ __global__ void __launch_bounds__(192, 1) fwd_kernel(const __grid_constant__ Fwd
           float2* gml = reinterpret_cast<float2*>(go + (size_t)ns * kMaxQV * HD);
           for (int i = et; i < nqv * (HD / 4); i += 128) {
             const int qv = i / (HD / 4), d4 = i % (HD / 4);
-            const float* src = part + qv * (HD + 2) + 4 * d4;
+            const float* src = part + qv * AttnCfg<HD, F::kAttnBufs>::kPartLd + 4 * d4;
             reinterpret_cast<float4*>(go + ((size_t)sp * kMaxQV + qv) * HD)[d4] =
                 make_float4(src[0], src[1], src[2], src[3]);
           }
           for (int qv = et; qv < nqv; qv += 128)
-            gml[sp * kMaxQV + qv] = make_float2(part[qv * (HD + 2) + HD], part[qv * (HD + 2) + HD + 1]);
+            gml[sp * kMaxQV + qv] = make_float2(part[qv * AttnCfg<HD, F::kAttnBufs>::kPartLd + HD],
+                                                 part[qv * AttnCfg<HD, F::kAttnBufs>::kPartLd + HD + 1]);
           epi_bar();
           if (et == 0) {
             const int old = atom_add_acq_rel(&f.attn_cnt[gidx], 1);  // publishes ours, acquires the others'

@@ -73,6 +73,9 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
   const uint32_t tmem = *tmem_slot;
   uint32_t armed[C::kStages];  // producer: times each ring slot was armed
   for (int s = 0; s < C::kStages; ++s) armed[s] = 0;
+  // ring slots this launch uses, and how many are filled before the PDL wait
+  const int R = (a.stages > 0 && a.stages < C::kStages) ? a.stages : C::kStages;
+  const int P = (a.pre_stages > 0 && a.pre_stages < R) ? a.pre_stages : R;
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -81,7 +84,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       for (int i = 0; i < kMaxSeg; ++i)
         if ((i < a.nseg || (a.pair && i < 2)) && !a.wpk[i]) tma_prefetch_desc(&a.wmap[i]);
       const int n = (int)(u1 - u0);
-      const int npre = n < C::kStages ? n : C::kStages;
+      const int npre = n < P ? n : P;
       // Unit cursor advanced incrementally: the producer issues one stage per
       // wake-up with no divisions on the path between the 'empty' signal and
       // the copies.
@@ -149,8 +152,8 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
       }
       pdl_wait();
       for (int i = 0; i < npre; ++i) issue_b(i, pre_kk[i], pre_tok[i]);
-      int s = npre % C::kStages;
-      uint32_t ph = (uint32_t)((npre / C::kStages) & 1) ^ 1u;
+      int s = npre % R;
+      uint32_t ph = (uint32_t)((npre / R) & 1) ^ 1u;
       for (int i = npre; i < n; ++i) {
         if (!mbar_wait(&empty[s], ph, abort_flag)) {
           set_status(a.status, ST_TIMEOUT_TMA);
@@ -162,7 +165,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
         issue_a(s);
         issue_b(s, kk, tok_tile);
         advance();
-        if (++s == C::kStages) { s = 0; ph ^= 1u; }
+        if (++s == R) { s = 0; ph ^= 1u; }
       }
       pdl_trigger();
     }
@@ -170,7 +173,8 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(kTileN, 2 * TT);
-      long i = 0;
+      int s = 0;          // ring slot of the next unit
+      uint32_t fph = 0;   // its 'full' phase parity
       int seg_i = 0;
       bool ok = true;
       for (long u = u0; u < u1 && ok;) {
@@ -181,9 +185,8 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
         if (!mbar_wait(&acce[ab], aph, abort_flag)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d = tmem + ab * C::kAccCols;
-        for (; u < ue; ++u, ++i) {
-          const int s = (int)(i % C::kStages);
-          if (!mbar_wait(&full[s], (uint32_t)((i / C::kStages) & 1), abort_flag)) { ok = false; break; }
+        for (; u < ue; ++u) {
+          if (!mbar_wait(&full[s], fph, abort_flag)) { ok = false; break; }
           tc_fence_after();
           const uint64_t ad = sw128_desc(smem_u32(sA + s * C::kABytes));
           const uint64_t bd = sw128_desc(smem_u32(sB + s * C::kBBytes));
@@ -191,6 +194,7 @@ __global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ Ge
           for (int k = 0; k < kChunkK / 16; ++k)
             umma_bf16(d, ad + 2 * k, bd + 2 * k, idesc, (u > ub || k > 0) ? 1u : 0u);
           umma_commit(&empty[s]);
+          if (++s == R) { s = 0; fph ^= 1u; }
         }
         if (!ok) break;
         umma_commit(&accf[ab]);

@@ -48,6 +48,8 @@ struct GemmArgs {
   float* partials;
   int* counters;
   uint32_t* status;
+  int stages;                 // ring slots used (0: all the kernel has)
+  int pre_stages;             // slots filled before waiting on the previous kernel (0: stages)
   // RMS row scale applied after the reduction (null: none)
   const float* ssq_in;
   int ssq_tiles;
