@@ -332,23 +332,7 @@ GemmArgs gemm_base(pard_ctx* c, int rows_cap, int tt) {
   return a;
 }
 
-// Ring depth of a launch and how much of it is filled before the PDL wait.
-// Weights do not depend on the previous kernel, so a deeper pre-wait fill
-// covers more of the hand-off between kernels; but it also competes with
-// the previous kernel's tail, which only pays for matrices much larger than
-// what the GPU's rings hold at the default depth.
-constexpr double kDeepMB = 40.0;
-constexpr int kRingDeep = 8, kPreDeep = 8, kRingShallow = 5, kPreShallow = 5;
-static void gemm_depth(GemmArgs& a, int tt) {
-  if (tt != 16) return;
-  const double mb = (double)a.w_tiles * a.kc * kTileN * kChunkK * 2 / 1e6;
-  const bool deep = mb >= kDeepMB;
-  a.stages = deep ? kRingDeep : kRingShallow;
-  a.pre_stages = deep ? kPreDeep : kPreShallow;
-}
-
 void run_gemm(pard_ctx* c, GemmArgs& a, int tt, cudaStream_t s) {
-  gemm_depth(a, tt);
   const long U = (long)a.w_tiles * a.tok_tiles * a.kc;
   const int grid = (int)std::min<long>(c->sm, U);
   launch_gemm(a, tt, grid, s, true);

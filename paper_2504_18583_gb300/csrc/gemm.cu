@@ -31,7 +31,8 @@
 namespace pard {
 
 template <int TT>
-__global__ void __launch_bounds__(192, 1) gemm_kernel(const __grid_constant__ GemmArgs a) {
+// two CTAs per SM at the 16-token tile: this launch's and the next one's
+__global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __grid_constant__ GemmArgs a) {
   using C = GemmCfg<TT>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));

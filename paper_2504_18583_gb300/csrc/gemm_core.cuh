@@ -15,7 +15,11 @@ struct GemmCfg {
   static constexpr int kABytes = kTileN * 128;       // 128 rows x 64 bf16
   static constexpr int kBBytes = 2 * TT * 128;       // 2*TT rows x 64 bf16
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStages = TT <= 16 ? 10 : (TT <= 32 ? 4 : 3);  // ring capacity (a launch may use fewer)
+  // Ring capacity (a launch may use fewer).  At the 16-token tile the CTA
+  // (about 106 KB of shared memory, at most 168 registers a thread) leaves
+  // room on its SM for one CTA of the next launch, which then starts, fills
+  // its ring and reaches its PDL wait while this one finishes.
+  static constexpr int kStages = TT <= 16 ? 5 : (TT <= 32 ? 4 : 3);
   static constexpr int kAccCols = 2 * TT;
   static constexpr int kNumAcc = (2 * kAccCols <= 256) ? 2 : 1;
   static constexpr int kTmemCols = kNumAcc * kAccCols <= 32 ? 32 : kNumAcc * kAccCols <= 64 ? 64
