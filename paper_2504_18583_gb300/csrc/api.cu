@@ -334,7 +334,9 @@ GemmArgs gemm_base(pard_ctx* c, int rows_cap, int tt) {
 
 void run_gemm(pard_ctx* c, GemmArgs& a, int tt, cudaStream_t s) {
   const long U = (long)a.w_tiles * a.tok_tiles * a.kc;
-  const int grid = (int)std::min<long>(c->sm, U);
+  // at least 8 units (128 KB of weights) a CTA: with fewer, the split-K
+  // finish of a tile gathers partials from too many CTAs
+  const int grid = (int)std::min<long>(c->sm, std::max<long>(1, U / 8));
   launch_gemm(a, tt, grid, s, true);
   c->launches++;
 }
