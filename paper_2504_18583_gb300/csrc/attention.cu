@@ -95,29 +95,42 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
     cluster_arrive();
     bool ok = my_n == 0 || mbar_wait(&s_recv, 0, &s_flag);
     if (!ok && threadIdx.x == 0) set_status(a.status, ST_TIMEOUT_EPI);
+    // every copy out of this CTA's partial has been read (its issuers waited
+    // before the barrier below), so the partial's area is free for the weights
     ok = __syncthreads_and(ok);
     if (ok) {
+      // split weights exp(m_s - max) / L of each finished row: a half-warp per
+      // row, lane s holding split s, max and sum by shuffles
+      float* sw = part;  // [my_n][kMaxCluster]
+      const int sr = threadIdx.x & 15;
+      for (int r0 = 0; r0 < my_n; r0 += kAttnThreads / 16) {
+        const int r = r0 + (int)(threadIdx.x >> 4);
+        const bool live = r < my_n && sr < (int)NS;
+        const float m = live ? recv[((size_t)sr * cnt + r) * LD + HD] : -INFINITY;
+        float mx = m;
+#pragma unroll
+        for (int off = 8; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off, 16));
+        const float w = m == -INFINITY ? 0.f : expf(m - mx);
+        float L = live ? recv[((size_t)sr * cnt + r) * LD + HD + 1] * w : 0.f;
+#pragma unroll
+        for (int off = 8; off > 0; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off, 16);
+        if (live) sw[r * kMaxCluster + sr] = w / L;
+      }
+      __syncthreads();
       for (int i = threadIdx.x; i < my_n * (HD / 4); i += kAttnThreads) {
         const int r = i / (HD / 4), d4 = i % (HD / 4);
-        float mx = -INFINITY;
-        for (int sr = 0; sr < (int)NS; ++sr) mx = fmaxf(mx, recv[((size_t)sr * cnt + r) * LD + HD]);
-        float L = 0.f;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int sr = 0; sr < (int)NS; ++sr) {
-          const float* src = recv + ((size_t)sr * cnt + r) * LD;
-          const float m = src[HD];
-          const float w = m == -INFINITY ? 0.f : expf(m - mx);
-          L += src[HD + 1] * w;
-          const float4 v = *reinterpret_cast<const float4*>(src + 4 * d4);
+#pragma unroll 4
+        for (int s2 = 0; s2 < (int)NS; ++s2) {
+          const float w = sw[r * kMaxCluster + s2];
+          const float4 v = *reinterpret_cast<const float4*>(recv + ((size_t)s2 * cnt + r) * LD + 4 * d4);
           acc.x += v.x * w;
           acc.y += v.y * w;
           acc.z += v.z * w;
           acc.w += v.w * w;
         }
-        const float inv = 1.0f / L;
         const int qv = my0 + r;
-        store_pair4(a.x_out, row0 + qv / GROUP, (kvh * GROUP + qv % GROUP) * HD + 4 * d4, a.x_rows,
-                    make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv));
+        store_pair4(a.x_out, row0 + qv / GROUP, (kvh * GROUP + qv % GROUP) * HD + 4 * d4, a.x_rows, acc);
       }
     }
     // second barrier, wait: no peer copies into this CTA any more
