@@ -228,6 +228,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-steps", type=int, default=2)
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end generation (profiling runs)")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the planted-acceptance and autoregressive runs (profiling runs: the timed steps "
+                         "are then the last launches)")
     ap.add_argument("--persistent", action="store_true",
                     help="run draft / verify as one persistent kernel instead of one kernel per phase")
     ap.add_argument("--workload", default="8b_greedy", choices=["8b_greedy", "8b_sample", "8b_batch16"],
@@ -414,7 +417,7 @@ def main():
                 "note": "verify input = the target's greedy continuation with each candidate corrupted "
                         "with probability 1 - alpha (seeded); draft still runs every step"}
 
-    headline = args.workload == "8b_greedy" and not args.layers
+    headline = args.workload == "8b_greedy" and not args.layers and not args.no_extras
     planted = planted_run(0.90, 24) if headline else None
 
     # autoregressive baseline on the same kernels: the target alone, one token
