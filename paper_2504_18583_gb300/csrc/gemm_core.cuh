@@ -555,10 +555,11 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
     for (int ch = 0; ch < C::kChunks; ++ch) {
       uint32_t r[32];
       tmem_ld32(tbase + ch * 32, r);
-      float4* dst = reinterpret_cast<float4*>(mine + ((size_t)ch * kTileN + fr) * kEpiTok);
+      // [chunk][j4][row] float4s: a warp's accesses are 512 contiguous bytes
+      float4* dst = reinterpret_cast<float4*>(mine + (size_t)ch * kTileN * kEpiTok) + fr;
 #pragma unroll
       for (int j4 = 0; j4 < 4; ++j4)
-        dst[j4] = make_float4(__uint_as_float(r[8 * j4 + 0]) + __uint_as_float(r[8 * j4 + 1]),
+        dst[j4 * kTileN] = make_float4(__uint_as_float(r[8 * j4 + 0]) + __uint_as_float(r[8 * j4 + 1]),
                               __uint_as_float(r[8 * j4 + 2]) + __uint_as_float(r[8 * j4 + 3]),
                               __uint_as_float(r[8 * j4 + 4]) + __uint_as_float(r[8 * j4 + 5]),
                               __uint_as_float(r[8 * j4 + 6]) + __uint_as_float(r[8 * j4 + 7]));
@@ -606,19 +607,19 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
     float v[kEpiTok];
 #pragma unroll
     for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
-    const size_t off = ((size_t)ch * kTileN + fr) * kEpiTok;
+    const size_t off = (size_t)ch * kTileN * kEpiTok;
     for (int k = 0; k < n_other; ++k) {
       float4 pv[4];
       if (staged) {
-        const float4* p = reinterpret_cast<const float4*>(ring + (size_t)k * kTileF + off);
+        const float4* p = reinterpret_cast<const float4*>(ring + (size_t)k * kTileF + off) + fr;
 #pragma unroll
-        for (int j4 = 0; j4 < 4; ++j4) pv[j4] = p[j4];
+        for (int j4 = 0; j4 < 4; ++j4) pv[j4] = p[j4 * kTileN];
       } else {
         const long cc = cf + 1 + k;
         const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
-        const float4* p = reinterpret_cast<const float4*>(a.partials + ((size_t)cc * 2 + sl) * kTileF + off);
+        const float4* p = reinterpret_cast<const float4*>(a.partials + ((size_t)cc * 2 + sl) * kTileF + off) + fr;
 #pragma unroll
-        for (int j4 = 0; j4 < 4; ++j4) pv[j4] = __ldcg(p + j4);
+        for (int j4 = 0; j4 < 4; ++j4) pv[j4] = __ldcg(p + j4 * kTileN);
       }
 #pragma unroll
       for (int j4 = 0; j4 < 4; ++j4) {
