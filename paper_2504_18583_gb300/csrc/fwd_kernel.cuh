@@ -37,7 +37,9 @@ struct FwdCfg {
   static constexpr int kAttnBufs = 3;  // K/V chunk ring (2 chunks in flight)
   static constexpr int kAttn = (AttnCfg<HD, kAttnBufs>::kSmem + 1023) / 1024 * 1024;
   static constexpr int kPhase = (int)((sizeof(Phase) + 127) / 128 * 128);  // epilogue's copy of its phase
-  static constexpr int kBar = 8 * (2 * kFwdStages + 5);  // full, empty, accf x2, acce x2, drain
+  // full, empty, accf x2, acce x2, drain; rounded to 16 bytes so that the
+  // epilogue scratch after it takes 16-byte vector accesses
+  static constexpr int kBar = (8 * (2 * kFwdStages + 5) + 15) / 16 * 16;
   static constexpr int kMisc = 64;
   static constexpr int kEpiFloats = Gm::kScratchFloats;
   static constexpr int kSmall = (kMaxQV + kMaxQV * kFwdMaxSplit) * 4;
@@ -172,7 +174,7 @@ __global__ void __launch_bounds__(192, 1) fwd_kernel(const __grid_constant__ Fwd
   uint64_t* accf = empty + S;
   uint64_t* acce = accf + 2;
   uint64_t* drain = acce + 2;
-  uint32_t* misc = reinterpret_cast<uint32_t*>(drain + 1);
+  uint32_t* misc = reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(full) + F::kBar);
   uint32_t* tmem_slot = misc;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
   int* bcast = reinterpret_cast<int*>(misc + 2);
