@@ -228,6 +228,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-steps", type=int, default=2)
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end generation (profiling runs)")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override the workload's batch (batch sweep; prompts keep the workload's length rule)")
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the planted-acceptance and autoregressive runs (profiling runs: the timed steps "
                          "are then the last launches)")
@@ -258,6 +260,8 @@ def main():
     if args.layers:
         wl = wl.replace(target=wl.target.replace(n_layers=args.layers),
                         draft=wl.draft.replace(n_layers=min(args.layers, wl.draft.n_layers)))
+    if args.batch:
+        wl = wl.replace(batch=args.batch)
     if args.warmup + args.steps > wl.n_new - 2:
         raise SystemExit(f"warmup + steps must stay below the generation length ({wl.n_new})")
     keep_host = rank == 0 and not args.no_cpu_baseline
@@ -417,7 +421,7 @@ def main():
                 "note": "verify input = the target's greedy continuation with each candidate corrupted "
                         "with probability 1 - alpha (seeded); draft still runs every step"}
 
-    headline = args.workload == "8b_greedy" and not args.layers and not args.no_extras
+    headline = args.workload == "8b_greedy" and not args.layers and not args.no_extras and not args.batch
     planted = planted_run(0.90, 24) if headline else None
 
     # autoregressive baseline on the same kernels: the target alone, one token
@@ -445,6 +449,39 @@ def main():
     if planted and ar:
         planted["speedup_vs_autoregressive"] = planted["value"] / ar["value"]
 
+    # vanilla speculative decoding on the same kernels: K sequential draft
+    # passes per iteration (K T_D + T_T against PARD's T_D + T_T)
+    def vsd_run(n_steps: int, warm: int = 3):
+        eng.prefill(prompts, wl.n_new, wl.K)
+        out = eng.alloc_step_outputs()
+        for i in range(warm):
+            eng.step(out, step=i + 1, sequential=True)
+        n_emit = torch.zeros(n_steps, dtype=torch.int32, device="cuda")
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(n_steps)]
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(n_steps):
+            ev[i][0].record(stream)
+            eng.draft_sequential(out, False, 1.0, 0, warm + i + 1)
+            ev[i][1].record(stream)
+            eng.verify(out, None, 1.0)
+            eng.accept_commit(out, False, 1.0, 0, warm + i + 1)
+            n_emit[i:i + 1].copy_(out["n_emit"][:1])
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        toks = int(n_emit.sum().item())
+        return {"value": toks / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms / n_steps,
+                "draft_ms": statistics.median(e[0].elapsed_time(e[1]) for e in ev), "steps": n_steps,
+                "note": "pard_draft_sequential (K draft forwards of one row each after the pending tokens) + "
+                        "verify + accept, on the same kernels"}
+
+    vsd = vsd_run(12) if headline else None
+    if vsd and planted:
+        # same candidates, so the same tokens per step: the ratio of step times
+        planted["speedup_vs_vanilla_sd"] = vsd["ms_per_step"] / planted["ms_per_step"]
+
     # roofline of the verify pass
     peak, peak_kind = peaks()
     ver_ms = statistics.median(phases["verify"])
@@ -471,7 +508,9 @@ def main():
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights and prompt ids)",
-        "config": {"workload": (args.workload + ": " + WORKLOAD_DESCS[args.workload]), "parallelism": f"replicas{ws}",
+        "config": {"workload": (args.workload + ": " + WORKLOAD_DESCS[args.workload]
+                                + (f" (batch overridden to {wl.batch})" if args.batch else "")),
+                   "batch": wl.batch, "parallelism": f"replicas{ws}",
                    "l2": "inputs larger than L2: 17.5 GB of weights stream from HBM every step",
                    "acceptance": "random-init draft: ~0 candidates accepted, ~1 token per step",
                    "forward_pass": "persistent" if fused_used else "per_phase"},
@@ -481,7 +520,7 @@ def main():
                      "achieved": ver_gbs, "peak": peak, "unit": "GB/s", "frac": ver_gbs / peak,
                      "peak_kind": peak_kind,
                      "traffic": (measured_verify_traffic(fused_used)
-                                 if args.workload == "8b_greedy" and not args.layers else None),
+                                 if args.workload == "8b_greedy" and not args.layers and not args.batch else None),
                      "traffic_source": "profiles/verify_pass_dram_traffic_8b.json (ncu DRAM bytes, 2-layer capture "
                                        "scaled to 32 layers; null if the kernels changed since)",
                      "bytes_per_launch": vb,
@@ -490,6 +529,7 @@ def main():
         "draft_roofline": {"achieved": dr_gbs, "frac": dr_gbs / peak, "bytes": db},
         "planted_acceptance": planted,
         "autoregressive_baseline": ar,
+        "vanilla_sd_baseline": vsd,
         "projection": {"alpha": alpha, "tokens_per_step": tok_per_step_proj,
                        "tokens_per_s": tok_per_step_proj / (step_ms / 1e3),
                        "note": "acceptance rate from the paper (context); same measured step time"},

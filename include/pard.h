@@ -133,6 +133,20 @@ pard_status pard_prefill(pard_ctx* ctx, const int32_t* d_tokens, const int32_t* 
 pard_status pard_draft(pard_ctx* ctx, int32_t sample, float temperature, uint64_t seed, uint64_t step,
                        int32_t* d_draft_out, float* d_draft_logits, void* stream);
 
+/* Vanilla speculative decoding's drafting stage (Section 2.2: the draft
+ * model produces the K candidates autoregressively; Section 3.1's
+ * autoregressive factorization), on the same kernels: K draft forwards,
+ * pass 0 over the pending real tokens (candidate 0 read at the last row),
+ * pass i >= 1 over candidate i-1 alone at position n-1+i.  Same arguments,
+ * outputs, sampling streams (Philox stream 0, row i for candidate i) and
+ * errors as pard_draft, and the same commit afterwards (the pending tokens
+ * are fed again next step), so pard_verify / pard_accept_commit follow it
+ * unchanged.  Per iteration it costs K draft forwards against PARD's one:
+ * the comparison of the paper's two iteration times, K*T_D + T_T and
+ * T_D + T_T. */
+pard_status pard_draft_sequential(pard_ctx* ctx, int32_t sample, float temperature, uint64_t seed, uint64_t step,
+                                  int32_t* d_draft_out, float* d_draft_logits, void* stream);
+
 /* One target forward over [last token, d_0..d_{K-1}] at positions
  * n-1..n+K-1 of each sequence.  d_draft_in [B][K]: candidates to verify, or
  * NULL for the ones the last pard_draft produced.  Writes per-row logit

@@ -19,6 +19,12 @@ Follows the paper's statement of the method:
   slots are dropped by length.  Draft KV of accepted candidates was computed
   from mask tokens, so those tokens are re-fed to the draft next step.
 * Autoregressive greedy decoding (Eq. 2) is the lossless reference.
+* Vanilla speculative decoding (Section 2.2, drafting stage; the
+  autoregressive factorization of Section 3.1): the same draft model
+  produces the K candidates one forward pass at a time, pass i feeding
+  candidate i-1 at the next position; verification, acceptance and commit are
+  unchanged.  Its per-iteration time is K * T_D + T_T against T_D + T_T for
+  PARD (Section 2.2).
 
 Readings where the paper is silent are listed in the repository's design
 notes; the ones that change numbers are: argmax takes the lowest index on
@@ -145,16 +151,18 @@ def accept_sampling(d: Sequence[int], z: np.ndarray, y: np.ndarray, temperature:
     return K, [int(x) for x in d] + [sample_gumbel_max(zK, seed, STREAM_BONUS, step, b, 0)]
 
 
+def draft_token(zi: np.ndarray, i: int, sample: bool, temperature: float, seed: int, step: int, b: int) -> int:
+    """Candidate i: argmax z_i (greedy) or a draw from softmax(z_i / T) by
+    Gumbel-max with the draft stream's uniforms of row i."""
+    if not sample:
+        return argmax_lowest(zi)
+    zt = (np.asarray(zi, dtype=np.float32) / np.float32(temperature)).astype(np.float32)
+    return sample_gumbel_max(zt, seed, STREAM_DRAFT, step, b, i)
+
+
 def draft_tokens(z: np.ndarray, sample: bool, temperature: float, seed: int, step: int, b: int) -> List[int]:
     """d_i = argmax z_i (greedy) or a draw from softmax(z_i / T) by Gumbel-max."""
-    out = []
-    for i in range(z.shape[0]):
-        if not sample:
-            out.append(argmax_lowest(z[i]))
-        else:
-            zi = (np.asarray(z[i], dtype=np.float32) / np.float32(temperature)).astype(np.float32)
-            out.append(sample_gumbel_max(zi, seed, STREAM_DRAFT, step, b, i))
-    return out
+    return [draft_token(z[i], i, sample, temperature, seed, step, b) for i in range(z.shape[0])]
 
 
 # --------------------------------------------------------------------------
@@ -246,6 +254,34 @@ class OracleDecoder:
             d[b] = draft_tokens(zb, wl.sample, wl.temperature, seed, step, b)
         return d, z
 
+    def draft_sequential(self, step: int, seed: int = 0,
+                         feed: Optional[np.ndarray] = None) -> Tuple[np.ndarray, np.ndarray]:
+        """Vanilla speculative decoding's drafting stage: K forward passes of
+        the draft model; pass 0 feeds the pending real tokens and reads its
+        last row, pass i >= 1 feeds candidate i-1 at position n-1+i.  The
+        draft cache keeps what the passes wrote; commit rolls it back by
+        length exactly as for the parallel draft (the pending tokens are fed
+        again next step).  feed [B,K] (teacher forcing): pass i >= 1 feeds
+        feed[b, i-1] instead of the oracle's own candidate.  Returns d [B,K],
+        z [B,K,V]."""
+        wl, K = self.wl, self.K
+        V = wl.draft.vocab
+        d = np.zeros((wl.batch, K), dtype=np.int32)
+        z = np.zeros((wl.batch, K, V), dtype=np.float32)
+        for b in range(wl.batch):
+            if self.done[b]:
+                continue
+            pend = self.pending[b]
+            p, n = len(pend), self.n[b]
+            zi = self.D.forward(b, pend, list(range(n - p, n)), [p - 1])[0]
+            for i in range(K):
+                if i > 0:
+                    prev = int(d[b, i - 1]) if feed is None else int(feed[b, i - 1])
+                    zi = self.D.forward(b, [prev], [n - 1 + i], [0])[0]
+                z[b, i] = zi
+                d[b, i] = draft_token(zi, i, wl.sample, wl.temperature, seed, step, b)
+        return d, z
+
     def verify(self, d: np.ndarray) -> np.ndarray:
         """Target forward over [x_{n-1}, d_0..d_{K-1}] at positions n-1..n+K-1."""
         wl, K = self.wl, self.K
@@ -303,13 +339,15 @@ class OracleDecoder:
     def all_done(self) -> bool:
         return all(self.done)
 
-    def run(self, prompts, seed: int = 0, max_steps: int = 10 ** 6):
-        """Full generation; returns (generated tokens per sequence, trace)."""
+    def run(self, prompts, seed: int = 0, max_steps: int = 10 ** 6, sequential: bool = False):
+        """Full generation; returns (generated tokens per sequence, trace).
+        sequential: vanilla speculative decoding's K-pass draft instead of
+        the parallel one."""
         self.prefill(prompts, seed)
         trace = []
         step = 1
         while not self.all_done() and step <= max_steps:
-            d, z = self.draft(step, seed)
+            d, z = self.draft_sequential(step, seed) if sequential else self.draft(step, seed)
             y = self.verify(d)
             acc, em = self.accept(d, z, y, step, seed)
             slots, n_out = self.commit(acc, em)

@@ -982,6 +982,50 @@ pard_status pard_draft(pard_ctx* c, int32_t sample, float temperature, uint64_t 
   });
 }
 
+// Vanilla speculative decoding's drafting stage on the same kernels: K
+// forward passes of the draft model, pass i picking candidate i (one
+// embedding / layers / LM head / select sequence per pass).
+pard_status pard_draft_sequential(pard_ctx* c, int32_t sample, float temperature, uint64_t seed, uint64_t step,
+                                  int32_t* d_out, float* d_logits, void* stream) {
+  if (!c) return fail(PARD_ERR_ARG, "null context");
+  if (!c->prefilled) return fail(PARD_ERR_STATE, "pard_draft_sequential before pard_prefill (or after pard_unpack_weights)");
+  if (c->K == 0) return fail(PARD_ERR_STATE, "pard_draft_sequential with K = 0 (autoregressive decoding has no draft)");
+  if (sample && !(temperature > 0.f)) return fail(PARD_ERR_ARG, "temperature must be > 0 when sampling");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  c->launches = 0;
+  return guarded([&]() -> pard_status {
+    set_call(c, seed, step, temperature > 0.f ? temperature : 1.0f, sample, s);
+    Model& M = c->m[1];
+    const int keep = (sample || d_logits) ? 1 : 0;
+    for (int i = 0; i < c->K; ++i) {
+      // pass 0: the pending real tokens (at most K + 1 per sequence); then one row
+      const int per_seq = i == 0 ? c->K + 1 : 1;
+      const int rows_cap = c->batch * per_seq;
+      EmbedArgs e = embed_base(c, 1, EMB_DRAFT_SEQ);
+      e.seq_i = i;
+      launch_embed(e, rows_cap, s, true);
+      c->launches++;
+      run_layers(c, 1, rows_cap, c->batch, per_seq, M.page_table, s);
+      run_lm_head(c, 1, c->xd, 2 * c->D.MC, c->ssq, rows_cap, pick_tt(rows_cap), c->rp.m_dev,
+                  keep ? c->dlogits : nullptr, c->rp.row_out, c->rp.row_gi, c->rp.row_seq, c->stats_d, c->stats_id,
+                  STREAM_DRAFT, s);
+      SelectArgs sa;
+      std::memset(&sa, 0, sizeof(sa));
+      sa.mode = SEL_DRAFT_SEQ;
+      sa.seq_i = i;
+      sa.batch = c->batch; sa.K = c->K; sa.w_tiles = c->D.w_tiles; sa.m_cap = c->D.MC; sa.vocab = c->D.vocab;
+      sa.stats = c->stats_d; sa.stats_i = c->stats_id; sa.call = c->call; sa.st = c->st;
+      sa.seq_row0 = c->rp.seq_row0; sa.out = d_out;
+      launch_select(sa, s, true);
+      c->launches++;
+    }
+    if (d_logits)
+      CK(cudaMemcpyAsync(d_logits, c->dlogits, (size_t)c->batch * c->K * c->D.vocab * 4, cudaMemcpyDeviceToDevice, s));
+    c->last_draft_sampled = sample != 0;
+    return PARD_OK;
+  });
+}
+
 pard_status pard_verify(pard_ctx* c, const int32_t* d_draft_in, float temperature, float* d_logits_out,
                         void* stream) {
   if (!c) return fail(PARD_ERR_ARG, "null context");

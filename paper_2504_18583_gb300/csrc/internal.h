@@ -135,8 +135,9 @@ struct RowPlan {     // row layout of one forward pass
 };
 
 struct EmbedArgs {
-  int mode;          // EMB_PREFILL, EMB_DRAFT, EMB_VERIFY
+  int mode;          // EMB_PREFILL, EMB_DRAFT, EMB_VERIFY, EMB_DRAFT_SEQ
   int batch, K, mask_id, vocab, d;
+  int seq_i;         // EMB_DRAFT_SEQ: pass index i (0: the pending tokens; i > 0: candidate i-1)
   const __nv_bfloat16* embed;
   const __nv_bfloat16* gain0;  // first layer's attention-norm gain
   const int* tokens;           // prefill: this chunk's tokens
@@ -150,11 +151,12 @@ struct EmbedArgs {
   int m_cap;
   uint32_t* status;
 };
-enum { EMB_PREFILL = 0, EMB_DRAFT = 1, EMB_VERIFY = 2 };
+enum { EMB_PREFILL = 0, EMB_DRAFT = 1, EMB_VERIFY = 2, EMB_DRAFT_SEQ = 3 };
 
 struct SelectArgs {
-  int mode;          // SEL_DRAFT, SEL_FIRST, SEL_NORM_ONLY
+  int mode;          // SEL_DRAFT, SEL_FIRST, SEL_NORM_ONLY, SEL_DRAFT_SEQ
   int batch, K, w_tiles, m_cap, vocab;
+  int seq_i;         // SEL_DRAFT_SEQ: the candidate this pass picks
   const float4* stats;
   const int2* stats_i;
   const CallArgs* call;
@@ -164,7 +166,7 @@ struct SelectArgs {
   const int* plen;   // first token: prompt lengths
   int n_new;
 };
-enum { SEL_DRAFT = 0, SEL_FIRST = 1, SEL_NORM_ONLY = 2 };
+enum { SEL_DRAFT = 0, SEL_FIRST = 1, SEL_NORM_ONLY = 2, SEL_DRAFT_SEQ = 3 };
 
 struct AcceptArgs {
   int batch, K, w_tiles, m_cap, vocab;

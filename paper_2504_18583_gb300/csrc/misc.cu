@@ -31,6 +31,9 @@ namespace pard {
 //                   K-1 mask tokens, at positions n-p .. n+K-2; logits rows
 //                   are the last real row and every mask row;
 //   verify:         [last token, d_0..d_{K-1}] at positions n-1 .. n+K-1;
+//   sequential draft (vanilla speculative decoding), pass i: i = 0 feeds
+//                   the pending real tokens (logits row: the last), i > 0
+//                   feeds candidate d_{i-1} at position n-1+i;
 //   prefill:        a chunk of one sequence's prompt.
 // h = E[token]; x = h * g (hi/lo bf16 pairs); ssq[t][m] = sum of h^2 over
 // the 128 columns of tile t.
@@ -49,7 +52,9 @@ __global__ void __launch_bounds__(128) embed_kernel(const __grid_constant__ Embe
     } else {
       for (int b = 0; b < a.batch; ++b) {
         s_row0[b] = total;
-        total += a.mode == EMB_DRAFT ? a.st.pend_cnt[b] + a.K - 1 : a.K + 1;
+        total += a.mode == EMB_DRAFT       ? a.st.pend_cnt[b] + a.K - 1
+                 : a.mode == EMB_DRAFT_SEQ ? (a.seq_i == 0 ? a.st.pend_cnt[b] : 1)
+                                           : a.K + 1;
       }
       s_row0[a.batch] = total;
     }
@@ -75,6 +80,18 @@ __global__ void __launch_bounds__(128) embed_kernel(const __grid_constant__ Embe
           tok = j < p ? a.st.pend[b * (a.st.kmax + 1) + j] : a.mask_id;
           pos = n - p + j;
           if (j >= p - 1) { gi = j - (p - 1); out = b * a.K + gi; }
+        } else if (a.mode == EMB_DRAFT_SEQ) {
+          const int p = a.st.pend_cnt[b];
+          if (a.seq_i == 0) {
+            tok = a.st.pend[b * (a.st.kmax + 1) + j];
+            pos = n - p + j;
+            if (j == p - 1) { gi = 0; out = b * a.K; }
+          } else {
+            tok = a.st.d[b * a.st.kmax + a.seq_i - 1];
+            pos = n - 1 + a.seq_i;
+            gi = a.seq_i;
+            out = b * a.K + a.seq_i;
+          }
         } else {
           tok = j == 0 ? a.st.pend[b * (a.st.kmax + 1) + a.st.pend_cnt[b] - 1] : a.d_in[b * a.K + j - 1];
           if (j > 0) a.st.d[b * a.st.kmax + j - 1] = tok;
@@ -230,6 +247,10 @@ __global__ void __launch_bounds__(256) select_kernel(const __grid_constant__ Sel
   if (a.mode == SEL_FIRST) {
     b = blockIdx.x;
     m = b;
+  } else if (a.mode == SEL_DRAFT_SEQ) {
+    b = blockIdx.x;
+    i = a.seq_i;
+    m = i == 0 ? a.seq_row0[b] + a.st.pend_cnt[b] - 1 : b;
   } else {
     b = blockIdx.x / a.K;
     i = blockIdx.x % a.K;
@@ -250,14 +271,14 @@ __global__ void __launch_bounds__(256) select_kernel(const __grid_constant__ Sel
     return;
   }
   a.st.dnorm[b * a.st.kmax + i] = make_float2(r.mx, r.se);
-  if (a.mode == SEL_DRAFT) {
+  if (a.mode == SEL_DRAFT || a.mode == SEL_DRAFT_SEQ) {
     a.st.d[b * a.st.kmax + i] = tok;
     if (a.out) a.out[b * a.K + i] = tok;
   }
 }
 
 void launch_select(const SelectArgs& a, cudaStream_t s, bool pdl) {
-  const int grid = a.mode == SEL_FIRST ? a.batch : a.batch * a.K;
+  const int grid = (a.mode == SEL_FIRST || a.mode == SEL_DRAFT_SEQ) ? a.batch : a.batch * a.K;
   PARD_LAUNCH(select_kernel, grid, 256, 0, s, pdl, a);
 }
 

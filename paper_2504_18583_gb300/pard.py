@@ -60,6 +60,7 @@ def lib() -> ctypes.CDLL:
                                         vp, sz, vp, sz, vp, vp, vp]
         L.pard_prefill.argtypes = [vp, vp, vp, i32, i32, i32, i32, f32, u64, vp, vp]
         L.pard_draft.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp]
+        L.pard_draft_sequential.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp]
         L.pard_verify.argtypes = [vp, vp, f32, vp, vp]
         L.pard_accept_commit.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp, vp, vp]
         L.pard_set_logits.argtypes = [vp, vp, vp, vp, f32, vp]
@@ -80,7 +81,8 @@ def lib() -> ctypes.CDLL:
         L.pard_set_fused_pass.restype = ctypes.c_int
         L.pard_fused_pass_used.argtypes = [vp]
         L.pard_fused_pass_used.restype = i32
-        for name in ("pard_load_weights", "pard_prefill", "pard_draft", "pard_verify", "pard_accept_commit",
+        for name in ("pard_load_weights", "pard_prefill", "pard_draft", "pard_draft_sequential", "pard_verify",
+                     "pard_accept_commit",
                      "pard_set_logits", "pard_get_state", "pard_read_kv", "pard_last_status"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
@@ -214,6 +216,12 @@ class PardEngine:
         _check(lib().pard_draft(self.ctx, int(sample), temperature, seed, step, out["draft"].data_ptr(),
                                 _ptr(out.get("draft_logits")), self.stream.cuda_stream), "pard_draft")
 
+    def draft_sequential(self, out, sample=False, temperature=1.0, seed=0, step=0):
+        """Vanilla speculative decoding's K-pass draft (same outputs as draft())."""
+        _check(lib().pard_draft_sequential(self.ctx, int(sample), temperature, seed, step, out["draft"].data_ptr(),
+                                           _ptr(out.get("draft_logits")), self.stream.cuda_stream),
+               "pard_draft_sequential")
+
     def verify(self, out, draft_in=None, temperature=1.0):
         _check(lib().pard_verify(self.ctx, _ptr(draft_in), temperature, _ptr(out.get("logits")),
                                  self.stream.cuda_stream), "pard_verify")
@@ -224,10 +232,11 @@ class PardEngine:
                                         out["kv_slots"].data_ptr(), out["n_emit"].data_ptr(),
                                         self.stream.cuda_stream), "pard_accept_commit")
 
-    def step(self, out, sample=False, temperature=1.0, seed=0, step=0):
-        """One PARD step: draft, verify, accept/commit (K = 0: one autoregressive token, no draft)."""
+    def step(self, out, sample=False, temperature=1.0, seed=0, step=0, sequential=False):
+        """One PARD step: draft, verify, accept/commit (K = 0: one autoregressive token, no draft;
+        sequential: vanilla speculative decoding's K-pass draft)."""
         if self.K:
-            self.draft(out, sample, temperature, seed, step)
+            (self.draft_sequential if sequential else self.draft)(out, sample, temperature, seed, step)
         self.verify(out, None, temperature)
         self.accept_commit(out, sample, temperature, seed, step)
 

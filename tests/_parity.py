@@ -82,15 +82,21 @@ def check_token(gpu_tok: int, oracle_logits: np.ndarray, stats: dict, what: str)
             stats["excused_tokens"] += 1
 
 
-def greedy_step(P: Pair, step: int, inject=None):
-    """One teacher-forced greedy step; returns the GPU outputs."""
+def greedy_step(P: Pair, step: int, inject=None, sequential: bool = False):
+    """One teacher-forced greedy step; returns the GPU outputs.  sequential:
+    vanilla speculative decoding's K-pass draft on both sides."""
     torch = P.torch
     wl, K = P.wl, P.wl.K
     out = P.eng.alloc_step_outputs(want_logits=True)
-    P.eng.draft(out, False, 1.0, 0, step)
+    if sequential:
+        P.eng.draft_sequential(out, False, 1.0, 0, step)
+    else:
+        P.eng.draft(out, False, 1.0, 0, step)
     d_gpu = out["draft"].cpu().numpy()
     z_gpu = out["draft_logits"].cpu().numpy()
-    d_or, z_or = P.oracle.draft(step)
+    # the sequential draft feeds each candidate to the next pass: the oracle
+    # is fed the GPU's (teacher forcing), so near-tie choices do not diverge
+    d_or, z_or = P.oracle.draft_sequential(step, feed=d_gpu) if sequential else P.oracle.draft(step)
     for b in P.active():
         err = float(np.abs(z_gpu[b] - z_or[b]).max())
         P.stats["max_draft_logit_err"] = max(P.stats["max_draft_logit_err"], err)

@@ -65,6 +65,7 @@ def test_load_rejects_bad_shapes_before_touching_the_device():
     assert code == -2 and "multiple" in pard.pard_last_error()
     code = pard.lib().pard_draft(None, 0, 1.0, 0, 0, None, None, None)
     assert code == -1
+    assert pard.lib().pard_draft_sequential(None, 0, 1.0, 0, 0, None, None, None) == -1
     assert pard.lib().pard_set_fused_pass(None, 1) == -1
     assert pard.lib().pard_fused_pass_used(None) == 0
 

@@ -19,13 +19,13 @@ def built():
     _build.build()
 
 
-def run_greedy(P: Pair, max_steps=64, inject_fn=None):
+def run_greedy(P: Pair, max_steps=64, inject_fn=None, sequential=False):
     P.prefill()
     step = 1
     outs = []
     while not P.oracle.all_done() and step <= max_steps:
         inject = inject_fn(P, step) if inject_fn else None
-        outs.append(greedy_step(P, step, inject))
+        outs.append(greedy_step(P, step, inject, sequential))
         step += 1
     n, gen, done = P.eng.state()
     assert done == [1 if d else 0 for d in P.oracle.done]
@@ -48,6 +48,24 @@ def test_tiny_greedy_matches_oracle_every_step(fused):
     # the generated sequence equals autoregressive greedy decoding where margins are clear
     assert P.stats["excused_tokens"] <= P.stats["checked_tokens"] // 10
     print("stats", P.stats)
+
+
+def test_vanilla_sd_sequential_draft_matches_oracle_every_step():
+    """Vanilla speculative decoding (K sequential draft passes, Section 2.2)
+    on the same kernels: draft logits, candidates, accept lengths and slots
+    against the oracle's sequential draft, batch 2, ragged prompts; with the
+    target as its own draft every candidate but the last step's is accepted."""
+    wl = S.WORKLOADS["tiny"].replace(batch=2, prompt_len=None, prompt_len_range=(20, 45), n_new=24)
+    P = Pair(wl)
+    run_greedy(P, sequential=True)
+    assert P.oracle.all_done()
+    print("stats", P.stats)
+    wl2 = S.WORKLOADS["tiny"].replace(n_new=20, prompt_len=30)
+    P2 = Pair(wl2, draft_is_target=True)
+    outs = run_greedy(P2, sequential=True)
+    accs = [int(o["a"][0]) for o in outs]
+    assert max(accs) == wl2.K
+    print("accept lengths", accs, P2.stats)
 
 
 def test_tiny_greedy_jittered_norms_batch_ragged():

@@ -228,10 +228,10 @@ def test_extra_mask_changes_no_earlier_row(tiny):
     assert np.array_equal(outs[0], outs[1])
 
 
-def _greedy_equivalence(wl, tw, dw):
+def _greedy_equivalence(wl, tw, dw, sequential=False):
     pr = wl.prompts()
     dec = oracle.OracleDecoder(wl, tw, dw, wl.page_order(0), wl.page_order(1))
-    gen, trace = dec.run(pr)
+    gen, trace = dec.run(pr, sequential=sequential)
     for b in range(wl.batch):
         assert gen[b] == oracle.ar_greedy(wl.target, tw, pr[b], wl.n_new)
     return trace
@@ -250,6 +250,31 @@ def test_pard_greedy_equals_ar_with_accepting_draft(tiny):
     trace = _greedy_equivalence(wl, tw, tw)
     accs = [a for t in trace for a in t["acc"]]
     assert min(accs[:len(trace)]) >= 1 and max(accs) >= 1
+
+
+def test_vanilla_sd_greedy_equals_autoregressive_greedy(tiny):
+    """Vanilla speculative decoding (K sequential draft passes) is lossless
+    too: greedy output equals the target's autoregressive greedy decode."""
+    wl, tw, dw = tiny
+    _greedy_equivalence(wl, tw, dw, sequential=True)
+
+
+def test_vanilla_sd_candidates_are_the_drafts_own_greedy_continuation(tiny):
+    """Greedy vanilla SD's candidates are the draft model's autoregressive
+    greedy continuation of the accepted prefix (Section 3.1's factorization),
+    here checked against Eq. 2 run on the draft model alone; and with the
+    target as its own draft every candidate is accepted."""
+    wl, tw, dw = tiny
+    pr = wl.prompts()
+    dec = oracle.OracleDecoder(wl, tw, dw, wl.page_order(0), wl.page_order(1))
+    first = dec.prefill(pr)
+    d, _ = dec.draft_sequential(1)
+    for b in range(wl.batch):
+        cont = oracle.ar_greedy(wl.draft, dw, list(pr[b]) + [first[b]], wl.K)
+        assert [int(x) for x in d[b]] == cont
+    wl2 = wl.replace(draft=wl.target, n_new=20, batch=1)
+    trace = _greedy_equivalence(wl2, tw, tw, sequential=True)
+    assert all(a == wl2.K for t in trace[:-1] for a in t["acc"])
 
 
 def test_greedy_accept_rule_every_length():
