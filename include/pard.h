@@ -147,6 +147,13 @@ pard_status pard_draft(pard_ctx* ctx, int32_t sample, float temperature, uint64_
 pard_status pard_draft_sequential(pard_ctx* ctx, int32_t sample, float temperature, uint64_t seed, uint64_t step,
                                   int32_t* d_draft_out, float* d_draft_logits, void* stream);
 
+/* Per-offset mask ids for the parallel draft (Section 4.3 compares one
+ * shared mask id with distinct ones): mask m_k (k = 0 .. K-2) takes
+ * h_ids[k]; h_ids = NULL or n = 0 restores the draft config's shared
+ * mask_id.  n <= max_k - 1, ids in [0, draft vocab); a later pard_draft
+ * with K - 1 > n returns PARD_ERR_STATE.  Synchronises `stream`. */
+pard_status pard_set_mask_ids(pard_ctx* ctx, const int32_t* h_ids, int32_t n, void* stream);
+
 /* One target forward over [last token, d_0..d_{K-1}] at positions
  * n-1..n+K-1 of each sequence.  d_draft_in [B][K]: candidates to verify, or
  * NULL for the ones the last pard_draft produced.  Writes per-row logit

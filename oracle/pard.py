@@ -3,8 +3,10 @@
 Follows the paper's statement of the method:
 
 * Parallel draft (Section 3.1, Eq. 6): the draft model reads the accepted
-  prefix followed by mask tokens m_0..m_{K-2} (one shared id, Section 4.3
-  "Shared Mask Token ID") and predicts x_n..x_{n+K-1} in one forward pass;
+  prefix followed by mask tokens m_0..m_{K-2} (one shared id by default,
+  Section 4.3 "Shared Mask Token ID"; one id per offset when mask_ids is set,
+  the alternative that section compares) and predicts x_n..x_{n+K-1} in one
+  forward pass;
   the prediction for x_{n+k} is read at the row holding m_{k-1} (k >= 1) or at
   the last real token (k = 0), so it conditions on x_0..x_{n-1}, m_0..m_{k-1}.
 * Verification (Section 2.2): one target forward over the last accepted
@@ -183,6 +185,7 @@ class OracleDecoder:
         self.T = OracleModel(wl.target, target_w, wl.batch, max_pos)
         self.D = OracleModel(wl.draft, draft_w, wl.batch, max_pos)
         self.mask_id = wl.draft.mask_id
+        self.mask_ids: Optional[List[int]] = None  # one id per mask offset (Section 4.3); None: shared
         n_pages = sum(self.reserve)
         po_t = page_order_t if page_order_t is not None else np.arange(n_pages, dtype=np.int32)
         po_d = page_order_d if page_order_d is not None else np.arange(n_pages, dtype=np.int32)
@@ -247,7 +250,8 @@ class OracleDecoder:
                 continue
             pend = self.pending[b]
             p, n = len(pend), self.n[b]
-            rows = list(pend) + [self.mask_id] * (K - 1)
+            masks = [self.mask_id] * (K - 1) if self.mask_ids is None else [int(x) for x in self.mask_ids[:K - 1]]
+            rows = list(pend) + masks
             pos = list(range(n - p, n + K - 1))
             zb = self.D.forward(b, rows, pos, [p - 1 + i for i in range(K)])
             z[b] = zb

@@ -128,7 +128,7 @@ struct WsOffsets {
   size_t row_tok, row_pos, row_seq, row_out, row_gi, seq_row0, m_dev;
   size_t g_row_seq, g_row_gi, g_m;
   size_t st_n, st_pc, st_pend, st_gen, st_max, st_done, st_d, st_dnorm, st_sa, st_snorm, st_spart, st_scnt;
-  size_t call, status, tmp_pos, pt[2], rope[2], g_plen, pack_tmp;
+  size_t call, status, tmp_pos, pt[2], rope[2], g_plen, pack_tmp, mask_ids;
   size_t fwd_tab, fwd_done, fwd_apart, fwd_acnt;
   size_t total;
 };
@@ -183,6 +183,7 @@ WsOffsets layout_ws(const Dims& D, const pard_limits& lim) {
   for (int mi = 0; mi < 2; ++mi) o.pt[mi] = L.take((size_t)B * D.pt_ld * 4);
   for (int mi = 0; mi < 2; ++mi) o.rope[mi] = L.take((size_t)D.pt_ld * lim.page_size * (D.hdmax / 2) * 8);
   o.g_plen = L.take((size_t)B * 4);
+  o.mask_ids = L.take((size_t)std::max(K, 1) * 4);
   o.pack_tmp = L.take(kPackTmpBytes);
   // persistent pass: 4 phase tables ([model][logits kept]), their completion
   // counters, and the attention split partials and arrival counters
@@ -284,6 +285,8 @@ struct pard_ctx {
   uint32_t* status;
   int* tmp_pos;
   int* g_plen;
+  int* mask_ids;          // per-offset draft mask ids (used when n_mask_ids > 0)
+  int n_mask_ids = 0;     // 0: the draft config's shared mask id
   // host state
   std::vector<int> order[2];
   int batch = 0, K = 0, n_new = 0;
@@ -621,6 +624,7 @@ EmbedArgs embed_base(pard_ctx* c, int mi, int mode) {
   const Model& M = c->m[mi];
   e.mode = mode;
   e.batch = c->batch; e.K = c->K; e.mask_id = M.cfg.mask_id; e.vocab = M.cfg.vocab; e.d = M.cfg.d_model;
+  e.mask_ids = c->n_mask_ids > 0 ? c->mask_ids : nullptr;
   e.embed = M.embed; e.gain0 = M.L[0].t[W_ATTN_NORM];
   e.st = c->st; e.rp = c->rp;
   e.h = c->h; e.x = c->xd; e.ssq = c->ssq; e.m_cap = c->D.MC; e.status = c->status;
@@ -747,6 +751,7 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
     c->st.samp_cnt = c->at<int>(o.st_scnt); c->st.kmax = lim->max_k;
     c->call = c->at<CallArgs>(o.call); c->status = c->at<uint32_t>(o.status);
     c->tmp_pos = c->at<int>(o.tmp_pos); c->g_plen = c->at<int>(o.g_plen);
+    c->mask_ids = c->at<int>(o.mask_ids);
     for (int mi = 0; mi < 2; ++mi)
       for (int kl = 0; kl < 2; ++kl) {
         const size_t t = (size_t)(2 * mi + kl) * c->D.fwd_phases;
@@ -950,6 +955,8 @@ pard_status pard_draft(pard_ctx* c, int32_t sample, float temperature, uint64_t 
   if (!c) return fail(PARD_ERR_ARG, "null context");
   if (!c->prefilled) return fail(PARD_ERR_STATE, "pard_draft before pard_prefill (or after pard_unpack_weights)");
   if (c->K == 0) return fail(PARD_ERR_STATE, "pard_draft with K = 0 (autoregressive decoding has no draft pass)");
+  if (c->n_mask_ids > 0 && c->n_mask_ids < c->K - 1)
+    return fail(PARD_ERR_STATE, "fewer per-offset mask ids than the K - 1 mask rows of the draft");
   if (sample && !(temperature > 0.f)) return fail(PARD_ERR_ARG, "temperature must be > 0 when sampling");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   c->launches = 0;
@@ -1186,6 +1193,24 @@ pard_status pard_unpack_weights(pard_ctx* c, void* stream) {
 }
 
 int32_t pard_launch_count(pard_ctx* c) { return c ? c->launches : 0; }
+
+pard_status pard_set_mask_ids(pard_ctx* c, const int32_t* h_ids, int32_t n, void* stream) {
+  if (!c) return fail(PARD_ERR_ARG, "null context");
+  if (!h_ids || n == 0) {
+    c->n_mask_ids = 0;
+    return PARD_OK;
+  }
+  if (n < 0 || n > std::max(c->lim.max_k - 1, 0)) return fail(PARD_ERR_ARG, "mask id count outside [0, max_k - 1]");
+  for (int i = 0; i < n; ++i)
+    if (h_ids[i] < 0 || h_ids[i] >= c->m[1].cfg.vocab) return fail(PARD_ERR_ARG, "mask id outside the draft vocabulary");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return guarded([&]() -> pard_status {
+    CK(cudaMemcpyAsync(c->mask_ids, h_ids, (size_t)n * 4, cudaMemcpyHostToDevice, s));
+    CK(cudaStreamSynchronize(s));
+    c->n_mask_ids = n;
+    return PARD_OK;
+  });
+}
 
 pard_status pard_set_fused_pass(pard_ctx* c, int32_t enable) {
   if (!c) return fail(PARD_ERR_ARG, "null context");

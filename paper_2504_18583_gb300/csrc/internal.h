@@ -138,6 +138,7 @@ struct EmbedArgs {
   int mode;          // EMB_PREFILL, EMB_DRAFT, EMB_VERIFY, EMB_DRAFT_SEQ
   int batch, K, mask_id, vocab, d;
   int seq_i;         // EMB_DRAFT_SEQ: pass index i (0: the pending tokens; i > 0: candidate i-1)
+  const int* mask_ids;  // EMB_DRAFT: id of mask m_k per offset k (null: mask_id for all)
   const __nv_bfloat16* embed;
   const __nv_bfloat16* gain0;  // first layer's attention-norm gain
   const int* tokens;           // prefill: this chunk's tokens

@@ -28,8 +28,9 @@ namespace pard {
 // ---------------------------------------------------------------------------
 // Row plan + embedding.  One block per row of the pass (grid = row capacity).
 //   draft  (Eq. 6): sequence b feeds its pend_cnt pending real tokens, then
-//                   K-1 mask tokens, at positions n-p .. n+K-2; logits rows
-//                   are the last real row and every mask row;
+//                   K-1 mask tokens (one shared id, or one id per offset),
+//                   at positions n-p .. n+K-2; logits rows are the last real
+//                   row and every mask row;
 //   verify:         [last token, d_0..d_{K-1}] at positions n-1 .. n+K-1;
 //   sequential draft (vanilla speculative decoding), pass i: i = 0 feeds
 //                   the pending real tokens (logits row: the last), i > 0
@@ -77,7 +78,7 @@ __global__ void __launch_bounds__(128) embed_kernel(const __grid_constant__ Embe
         const int n = a.st.n[b];
         if (a.mode == EMB_DRAFT) {
           const int p = a.st.pend_cnt[b];
-          tok = j < p ? a.st.pend[b * (a.st.kmax + 1) + j] : a.mask_id;
+          tok = j < p ? a.st.pend[b * (a.st.kmax + 1) + j] : (a.mask_ids ? a.mask_ids[j - p] : a.mask_id);
           pos = n - p + j;
           if (j >= p - 1) { gi = j - (p - 1); out = b * a.K + gi; }
         } else if (a.mode == EMB_DRAFT_SEQ) {

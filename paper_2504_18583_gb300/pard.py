@@ -61,6 +61,7 @@ def lib() -> ctypes.CDLL:
         L.pard_prefill.argtypes = [vp, vp, vp, i32, i32, i32, i32, f32, u64, vp, vp]
         L.pard_draft.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp]
         L.pard_draft_sequential.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp]
+        L.pard_set_mask_ids.argtypes = [vp, vp, i32, vp]
         L.pard_verify.argtypes = [vp, vp, f32, vp, vp]
         L.pard_accept_commit.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp, vp, vp]
         L.pard_set_logits.argtypes = [vp, vp, vp, vp, f32, vp]
@@ -82,7 +83,7 @@ def lib() -> ctypes.CDLL:
         L.pard_fused_pass_used.argtypes = [vp]
         L.pard_fused_pass_used.restype = i32
         for name in ("pard_load_weights", "pard_prefill", "pard_draft", "pard_draft_sequential", "pard_verify",
-                     "pard_accept_commit",
+                     "pard_accept_commit", "pard_set_mask_ids",
                      "pard_set_logits", "pard_get_state", "pard_read_kv", "pard_last_status"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
@@ -221,6 +222,13 @@ class PardEngine:
         _check(lib().pard_draft_sequential(self.ctx, int(sample), temperature, seed, step, out["draft"].data_ptr(),
                                            _ptr(out.get("draft_logits")), self.stream.cuda_stream),
                "pard_draft_sequential")
+
+    def set_mask_ids(self, ids=None):
+        """One mask id per draft offset (None: the config's shared id)."""
+        n = 0 if ids is None else len(ids)
+        arr = (ctypes.c_int32 * max(n, 1))(*(ids or [0]))
+        _check(lib().pard_set_mask_ids(self.ctx, ctypes.cast(arr, ctypes.c_void_p) if n else None, n,
+                                       self.stream.cuda_stream), "pard_set_mask_ids")
 
     def verify(self, out, draft_in=None, temperature=1.0):
         _check(lib().pard_verify(self.ctx, _ptr(draft_in), temperature, _ptr(out.get("logits")),

@@ -68,6 +68,33 @@ def test_vanilla_sd_sequential_draft_matches_oracle_every_step():
     print("accept lengths", accs, P2.stats)
 
 
+def test_distinct_mask_ids_and_k12_match_oracle_every_step():
+    """One mask id per offset (Section 4.3's alternative to the shared id)
+    and K = 12 (verify 13 rows, draft up to 24 rows per sequence: two
+    attention row blocks), batch 2, against the oracle step by step; the
+    argument and state checks of pard_set_mask_ids."""
+    from paper_2504_18583_gb300 import pard
+    wl = S.WORKLOADS["tiny"].replace(K=12, batch=2, n_new=24, prompt_len=None, prompt_len_range=(20, 45))
+    V = wl.draft.vocab
+    ids = [V - 2 - k for k in range(wl.K - 1)]
+    P = Pair(wl)
+    P.eng.set_mask_ids(ids)
+    P.oracle.mask_ids = ids
+    run_greedy(P)
+    assert P.oracle.all_done()
+    print("stats", P.stats)
+    with pytest.raises(pard.PardError):
+        P.eng.set_mask_ids(list(range(wl.K)))       # more than max_k - 1 offsets
+    with pytest.raises(pard.PardError):
+        P.eng.set_mask_ids([V] + ids[1:])            # outside the vocabulary
+    P.eng.set_mask_ids(ids[:3])                      # too few for K - 1 = 11 mask rows
+    P.eng.prefill(P.prompts, wl.n_new, wl.K)
+    out = P.eng.alloc_step_outputs()
+    with pytest.raises(pard.PardError):
+        P.eng.draft(out)
+    P.eng.set_mask_ids(None)
+
+
 def test_tiny_greedy_jittered_norms_batch_ragged():
     """Batch of 3 with prompts 17 / 33 / 50 tokens (page boundaries at
     several offsets), norm gains != 1, prefill chunks of 64 rows."""

@@ -277,6 +277,36 @@ def test_vanilla_sd_candidates_are_the_drafts_own_greedy_continuation(tiny):
     assert all(a == wl2.K for t in trace[:-1] for a in t["acc"])
 
 
+def test_distinct_mask_ids_keep_pard_lossless_and_reach_the_draft(tiny):
+    """One mask id per offset (Section 4.3's alternative to the shared id):
+    greedy PARD still equals autoregressive greedy decoding, K = 12 (verify
+    13 rows, draft up to 24); and the mask rows' logits are the draft model's
+    forward over exactly those ids (they differ from the shared-id ones)."""
+    wl, tw, dw = tiny
+    wl = wl.replace(K=12, n_new=20, batch=2)
+    V = wl.draft.vocab
+    ids = [V - 2 - k for k in range(wl.K - 1)]
+    pr = wl.prompts()
+    dec = oracle.OracleDecoder(wl, tw, dw, wl.page_order(0), wl.page_order(1))
+    dec.mask_ids = ids
+    gen, _ = dec.run(pr)
+    for b in range(wl.batch):
+        assert gen[b] == oracle.ar_greedy(wl.target, tw, pr[b], wl.n_new)
+    dec2 = oracle.OracleDecoder(wl, tw, dw, wl.page_order(0), wl.page_order(1))
+    first = dec2.prefill(pr)
+    dec2.mask_ids = ids
+    _, z = dec2.draft(1)
+    m = P.OracleModel(wl.draft, dw, 1, 128)
+    P0 = len(pr[0])
+    m.forward(0, pr[0], range(P0), [])
+    ref = m.forward(0, [first[0]] + ids, range(P0, P0 + wl.K), range(wl.K))
+    assert np.array_equal(z[0], ref)
+    dec3 = oracle.OracleDecoder(wl, tw, dw, wl.page_order(0), wl.page_order(1))
+    dec3.prefill(pr)
+    _, z_shared = dec3.draft(1)
+    assert np.array_equal(z_shared[0, 0], z[0, 0]) and not np.array_equal(z_shared[0, 1:], z[0, 1:])
+
+
 def test_greedy_accept_rule_every_length():
     rng = np.random.default_rng(3)
     K, V = 5, 11
