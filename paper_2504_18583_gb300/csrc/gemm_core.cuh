@@ -18,8 +18,10 @@ struct GemmCfg {
   // Ring capacity (a launch may use fewer).  At the 16-token tile the CTA
   // (about 106 KB of shared memory, at most 168 registers a thread) leaves
   // room on its SM for one CTA of the next launch, which then starts, fills
-  // its ring and reaches its PDL wait while this one finishes.
-  static constexpr int kStages = TT <= 16 ? 5 : (TT <= 32 ? 4 : 3);
+  // its ring and reaches its PDL wait while this one finishes.  Wider tiles
+  // run one CTA per SM and take a deeper ring (~200 KB) instead: with 4 and
+  // 3 stages they kept too few weight bytes in flight per SM.
+  static constexpr int kStages = TT <= 16 ? 5 : (TT <= 32 ? 8 : 6);
   static constexpr int kAccCols = 2 * TT;
   static constexpr int kNumAcc = (2 * kAccCols <= 256) ? 2 : 1;
   static constexpr int kTmemCols = kNumAcc * kAccCols <= 32 ? 32 : kNumAcc * kAccCols <= 64 ? 64
@@ -535,15 +537,16 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
   using C = GemmCfg<TT>;
   constexpr int kTileF = kTileN * TT;  // floats of one partial tile
   if (ub == t * a.kc && ue == (t + 1) * a.kc) {
+    EpiPre pre = pre0;  // one chunk's loads live at a time
 #pragma unroll 1
     for (int ch = 0; ch < C::kChunks; ++ch) {
+      if (ch > 0) pre = epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M);
       uint32_t r[32];
       tmem_ld32(tbase + ch * 32, r);
       float v[kEpiTok];
 #pragma unroll
       for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
-      epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S,
-                ch == 0 ? pre0 : epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M));
+      epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S, pre);
     }
     return true;
   }
@@ -600,8 +603,10 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
     *abort_flag = 1;
     return false;
   }
+  EpiPre pre = pre0;
 #pragma unroll 1
   for (int ch = 0; ch < C::kChunks; ++ch) {
+    if (ch > 0) pre = epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M);
     uint32_t r[32];
     tmem_ld32(tbase + ch * 32, r);
     float v[kEpiTok];
@@ -629,8 +634,7 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
         v[4 * j4 + 3] += pv[j4].w;
       }
     }
-    epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S,
-              ch == 0 ? pre0 : epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M));
+    epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S, pre);
   }
   if (et == 0) a.counters[t] = 0;
   return true;
