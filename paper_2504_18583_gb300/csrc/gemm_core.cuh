@@ -536,10 +536,14 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
                                   volatile int* fx_armed, volatile int* abort_flag, int* bcast) {
   using C = GemmCfg<TT>;
   constexpr int kTileF = kTileN * TT;  // floats of one partial tile
+  // 16-token chunks holding at least one of the pass's M rows; the others are
+  // neither finished nor exchanged (their rows are not outputs)
+  const int nch = max(0, min(C::kChunks, (M - tok_base + kEpiTok - 1) / kEpiTok));
+  const int kChF = kTileN * kEpiTok;   // floats of one chunk of a partial tile
   if (ub == t * a.kc && ue == (t + 1) * a.kc) {
     EpiPre pre = pre0;  // one chunk's loads live at a time
 #pragma unroll 1
-    for (int ch = 0; ch < C::kChunks; ++ch) {
+    for (int ch = 0; ch < nch; ++ch) {
       if (ch > 0) pre = epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M);
       uint32_t r[32];
       tmem_ld32(tbase + ch * 32, r);
@@ -555,7 +559,7 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
     const int slot = (ub == u0) ? 0 : 1;
     float* mine = a.partials + ((size_t)c * 2 + slot) * kTileF;
 #pragma unroll 1
-    for (int ch = 0; ch < C::kChunks; ++ch) {
+    for (int ch = 0; ch < nch; ++ch) {
       uint32_t r[32];
       tmem_ld32(tbase + ch * 32, r);
       // [chunk][j4][row] float4s: a warp's accesses are 512 contiguous bytes
@@ -574,20 +578,21 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
     return true;
   }
   const int n_other = (int)(cl - cf);
-  const bool staged = (uint32_t)n_other * kTileF * 4 <= ring_bytes;
+  const uint32_t part_bytes = (uint32_t)nch * kChF * 4;  // of one contributor: its first nch chunks
+  const bool staged = (uint32_t)n_other * part_bytes <= ring_bytes;
   if (et == 0) {
     const bool ok = wait_count(&a.counters[t], n_other, abort_flag);
     if (!ok) set_status(a.status, ST_TIMEOUT_EPI);
-    if (ok && staged) {
+    if (ok && staged && nch > 0) {
       // the partials were written through the generic proxy; the copies read
       // them through the async proxy
       fence_proxy_async();
       *fx_armed = 1;
-      mbar_arrive_expect_tx(fx, (uint32_t)n_other * kTileF * 4);
+      mbar_arrive_expect_tx(fx, (uint32_t)n_other * part_bytes);
       for (int k = 0; k < n_other; ++k) {
         const long cc = cf + 1 + k;
         const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
-        bulk_load(ring + (size_t)k * kTileF, a.partials + ((size_t)cc * 2 + sl) * kTileF, kTileF * 4, fx);
+        bulk_load(ring + (size_t)k * nch * kChF, a.partials + ((size_t)cc * 2 + sl) * kTileF, part_bytes, fx);
       }
     }
     bcast[0] = ok ? 1 : 0;
@@ -597,7 +602,7 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
     *abort_flag = 1;
     return false;
   }
-  const bool late = staged && !mbar_wait(fx, 0, abort_flag);
+  const bool late = staged && nch > 0 && !mbar_wait(fx, 0, abort_flag);
   if (epi_bar_any(late)) {
     if (et == 0) set_status(a.status, ST_TIMEOUT_EPI);
     *abort_flag = 1;
@@ -605,7 +610,7 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
   }
   EpiPre pre = pre0;
 #pragma unroll 1
-  for (int ch = 0; ch < C::kChunks; ++ch) {
+  for (int ch = 0; ch < nch; ++ch) {
     if (ch > 0) pre = epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M);
     uint32_t r[32];
     tmem_ld32(tbase + ch * 32, r);
@@ -616,7 +621,7 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
     for (int k = 0; k < n_other; ++k) {
       float4 pv[4];
       if (staged) {
-        const float4* p = reinterpret_cast<const float4*>(ring + (size_t)k * kTileF + off) + fr;
+        const float4* p = reinterpret_cast<const float4*>(ring + (size_t)k * nch * kChF + off) + fr;
 #pragma unroll
         for (int j4 = 0; j4 < 4; ++j4) pv[j4] = p[j4 * kTileN];
       } else {
