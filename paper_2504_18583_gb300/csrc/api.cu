@@ -96,7 +96,6 @@ struct Dims {
   int dmax, qdmax, ffnmax, vocab, hkvmax, hdmax, w_tiles, pt_ld, sm;
   int ffn_pad;      // widest FFN rounded up to whole 64-column blocks
   int fwd_phases;   // phase capacity of one persistent-pass table (5 per layer + LM head)
-  size_t attn_part_floats;
 };
 
 int round_up(int x, int m) { return (x + m - 1) / m * m; }
@@ -116,7 +115,6 @@ Dims make_dims(const pard_model_cfg& t, const pard_model_cfg& d, const pard_limi
   D.w_tiles = (t.vocab + kTileN - 1) / kTileN;
   D.pt_ld = (lim.max_ctx + lim.page_size - 1) / lim.page_size;
   D.sm = sm;
-  D.attn_part_floats = 0;  // splits combine through distributed shared memory
   D.fwd_phases = 5 * std::max(t.n_layers, d.n_layers) + 1;
   return D;
 }
@@ -124,7 +122,7 @@ Dims make_dims(const pard_model_cfg& t, const pard_model_cfg& d, const pard_limi
 constexpr size_t kPackTmpBytes = (size_t)32 << 20;  // scratch for in-place weight packing
 
 struct WsOffsets {
-  size_t h, xd, xo, xf, xg, ssq, ssqg, q, gpart, gcnt, apart, acnt, stats_t, stats_it, stats_d, stats_id, logits, dlogits;
+  size_t h, xd, xo, xf, xg, ssq, ssqg, q, gpart, gcnt, stats_t, stats_it, stats_d, stats_id, logits, dlogits;
   size_t row_tok, row_pos, row_seq, row_out, row_gi, seq_row0, m_dev;
   size_t g_row_seq, g_row_gi, g_m;
   size_t st_n, st_pc, st_pend, st_gen, st_max, st_done, st_d, st_dnorm, st_sa, st_snorm, st_spart, st_scnt;
@@ -147,8 +145,6 @@ WsOffsets layout_ws(const Dims& D, const pard_limits& lim) {
   o.q = L.take((size_t)D.MC * D.qdmax * 4);
   o.gpart = L.take((size_t)D.sm * 2 * kTileN * 64 * 4);
   o.gcnt = L.take((size_t)65536 * 4);
-  o.apart = L.take(D.attn_part_floats * 4);
-  o.acnt = L.take((size_t)65536 * 4);
   o.stats_t = L.take((size_t)D.w_tiles * D.MC * 16);
   o.stats_it = L.take((size_t)D.w_tiles * D.MC * 8);
   o.stats_d = L.take((size_t)D.w_tiles * D.MC * 16);
@@ -273,9 +269,9 @@ struct pard_ctx {
   uint8_t* ws = nullptr;
   int sm = 0;
   // device views
-  float *h, *ssq, *ssqg, *q, *gpart, *apart, *logits, *dlogits;
+  float *h, *ssq, *ssqg, *q, *gpart, *logits, *dlogits;
   __nv_bfloat16 *xd, *xo, *xf, *xg;
-  int *gcnt, *acnt;
+  int* gcnt;
   float4 *stats_t, *stats_d;
   int2 *stats_it, *stats_id;
   RowPlan rp;
@@ -411,7 +407,7 @@ LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch
     a.row_blocks = geo.row_blocks; a.n_split = geo.n_split;
     a.scale = (float)(1.0 / std::sqrt((double)cf.head_dim));
     a.x_out = c->xo; a.x_rows = 2 * c->D.MC;
-    a.part = c->apart; a.counters = c->acnt; a.status = c->status;
+    a.status = c->status;
   }
   // O projection + residual; emits x = h * g_mlp and the new row sums of squares
   {
@@ -734,11 +730,11 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
     c->ws = reinterpret_cast<uint8_t*>(workspace);
     const WsOffsets& o = c->o;
     c->h = c->at<float>(o.h); c->ssq = c->at<float>(o.ssq); c->ssqg = c->at<float>(o.ssqg); c->q = c->at<float>(o.q);
-    c->gpart = c->at<float>(o.gpart); c->apart = c->at<float>(o.apart);
+    c->gpart = c->at<float>(o.gpart);
     c->logits = c->at<float>(o.logits); c->dlogits = c->at<float>(o.dlogits);
     c->xd = c->at<__nv_bfloat16>(o.xd); c->xo = c->at<__nv_bfloat16>(o.xo); c->xf = c->at<__nv_bfloat16>(o.xf);
     c->xg = c->at<__nv_bfloat16>(o.xg);
-    c->gcnt = c->at<int>(o.gcnt); c->acnt = c->at<int>(o.acnt);
+    c->gcnt = c->at<int>(o.gcnt);
     c->stats_t = c->at<float4>(o.stats_t); c->stats_it = c->at<int2>(o.stats_it);
     c->stats_d = c->at<float4>(o.stats_d); c->stats_id = c->at<int2>(o.stats_id);
     c->rp = RowPlan{c->at<int>(o.row_tok), c->at<int>(o.row_pos), c->at<int>(o.row_seq), c->at<int>(o.row_out),
@@ -763,7 +759,6 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
 
     // counters start at zero; the reduction kernels leave them at zero
     CK(cudaMemsetAsync(c->gcnt, 0, 65536 * 4, s));
-    CK(cudaMemsetAsync(c->acnt, 0, 65536 * 4, s));
     CK(cudaMemsetAsync(c->fwd_acnt, 0, (size_t)kFwdMaxAttnItems * 4, s));
     CK(cudaMemsetAsync(c->st.samp_cnt, 0, lim->max_batch * 4, s));
     CK(cudaMemsetAsync(c->status, 0, 4, s));

@@ -178,8 +178,6 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
   cluster_sync();  // peers may still be reading this CTA's partial
 }
 
-size_t attention_part_floats(int, int, int, int, int, int) { return 0; }
-
 template <int HD, int GROUP>
 static cudaError_t launch_attn_t(const AttnArgs& a, int grid, int cluster, cudaStream_t s, bool pdl) {
   static bool configured = false;

@@ -277,7 +277,6 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
 int gemm_smem_bytes(int tt) {
   switch (tt) {
     case 16: return GemmCfg<16>::kSmem;
-    case 32: return GemmCfg<32>::kSmem;
     case 64: return GemmCfg<64>::kSmem;
     default: return -1;
   }
@@ -309,7 +308,6 @@ void launch_gemm(const GemmArgs& a, int tt, int grid, cudaStream_t s, bool pdl) 
   cudaError_t e;
   switch (tt) {
     case 16: e = launch_tt<16>(a, grid, s, pdl); break;
-    case 32: e = launch_tt<32>(a, grid, s, pdl); break;
     default: e = launch_tt<64>(a, grid, s, pdl); break;
   }
   if (e != cudaSuccess) throw e;

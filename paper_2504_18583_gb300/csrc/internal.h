@@ -100,8 +100,6 @@ struct AttnArgs {
   float scale;
   __nv_bfloat16* x_out;       // packed [2*rows][hq*hd] hi/lo
   int x_rows;
-  float* part;                // split partials
-  int* counters;
   uint32_t* status;
 };
 
@@ -235,7 +233,6 @@ void launch_read_kv(const __nv_bfloat16* kc, const __nv_bfloat16* vc, const int*
 void launch_gemm(const GemmArgs& a, int tt, int grid, cudaStream_t s, bool pdl);
 int gemm_smem_bytes(int tt);
 void launch_attention(const AttnArgs& a, int grid_x, cudaStream_t s, bool pdl);
-size_t attention_part_floats(int batch, int hkv, int row_blocks, int n_split, int qv, int hd);
 int attention_rows_per_block(int group);
 
 }  // namespace pard
