@@ -123,6 +123,20 @@ class ClockSampler:
                 "reasons": sorted(reasons)}
 
 
+def aggregate_over_ranks(ms: float, toks: int, ws: int, device: str = "cuda"):
+    """Replicas: the job's time is the slowest rank's timed region, its tokens
+    the sum over ranks (every rank runs the whole workload on its own GPU)."""
+    if ws == 1:
+        return ms, toks
+    import torch
+    import torch.distributed as dist
+    t_ms = torch.tensor([ms], dtype=torch.float64, device=device)
+    t_tok = torch.tensor([float(toks)], dtype=torch.float64, device=device)
+    dist.all_reduce(t_ms, op=dist.ReduceOp.MAX)
+    dist.all_reduce(t_tok, op=dist.ReduceOp.SUM)
+    return float(t_ms[0]), int(t_tok[0])
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -315,6 +329,8 @@ def main():
             n_emit[i].copy_(out["n_emit"])
         ev[1].record(stream)
         torch.cuda.synchronize()
+        if ws > 1:
+            torch.distributed.barrier()
         ms = ev[0].elapsed_time(ev[1])
         phases = None
         if phase_events:
@@ -333,14 +349,7 @@ def main():
     fused_used = eng.fused_pass_used()
 
     # max over ranks
-    tot_toks = toks
-    ms_max = ms
-    if ws > 1:
-        t = torch.tensor([ms, float(toks)], dtype=torch.float64, device="cuda")
-        tmax = t.clone()
-        torch.distributed.all_reduce(tmax[:1], op=torch.distributed.ReduceOp.MAX)
-        torch.distributed.all_reduce(t[1:], op=torch.distributed.ReduceOp.SUM)
-        ms_max, tot_toks = float(tmax[0]), int(t[1])
+    ms_max, tot_toks = aggregate_over_ranks(ms, toks, ws)
     value = tot_toks / (ms_max / 1e3)
 
     # e2e: host prompt in (pinned), full generation, host tokens out each step
