@@ -199,6 +199,13 @@ pard_status pard_read_kv(pard_ctx* ctx, int32_t model, int32_t layer, int32_t b,
  * PARD_ERR_DEVICE_CHECK when bits are set. */
 pard_status pard_last_status(pard_ctx* ctx, uint32_t* h_flags, void* stream);
 
+/* Failure-path self test: enqueue one kernel whose bounded pipeline wait
+ * (the one every GEMM stage uses) waits on a barrier nothing completes; after
+ * the wait limit (2 s) it sets the timeout bit of the device status word
+ * (bit 0) and returns, leaving the context usable.  A following
+ * pard_last_status returns PARD_ERR_TIMEOUT with that bit. */
+pard_status pard_selftest_stalled_wait(pard_ctx* ctx, void* stream);
+
 /* Restore every matrix pard_load_weights packed to row-major order
  * (synchronises `stream`).  The context accepts no further decode calls. */
 pard_status pard_unpack_weights(pard_ctx* ctx, void* stream);

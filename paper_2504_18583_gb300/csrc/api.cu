@@ -1172,6 +1172,15 @@ pard_status pard_last_status(pard_ctx* c, uint32_t* h_flags, void* stream) {
   });
 }
 
+pard_status pard_selftest_stalled_wait(pard_ctx* c, void* stream) {
+  if (!c) return fail(PARD_ERR_ARG, "null context");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return guarded([&]() -> pard_status {
+    launch_stalled_wait(c->status, s);
+    return PARD_OK;
+  });
+}
+
 pard_status pard_unpack_weights(pard_ctx* c, void* stream) {
   if (!c) return fail(PARD_ERR_ARG, "null context");
   if (c->unpacked) return PARD_OK;

@@ -230,6 +230,7 @@ void launch_copy_f32(const float* src, float* dst, size_t n, cudaStream_t s, boo
 void launch_read_kv(const __nv_bfloat16* kc, const __nv_bfloat16* vc, const int* page_table_row, const int* pos, int n,
                     int hkv, int hd, int page_size, __nv_bfloat16* ok, __nv_bfloat16* ov, cudaStream_t s);
 
+void launch_stalled_wait(uint32_t* status, cudaStream_t s);
 void launch_gemm(const GemmArgs& a, int tt, int grid, cudaStream_t s, bool pdl);
 int gemm_smem_bytes(int tt);
 void launch_attention(const AttnArgs& a, int grid_x, cudaStream_t s, bool pdl);

@@ -132,6 +132,24 @@ __global__ void __launch_bounds__(128) embed_kernel(const __grid_constant__ Embe
   }
 }
 
+// Failure-path self test: one thread waits, through the pipelines' bounded
+// wait, on an mbarrier that nothing arrives on; the wait gives up after its
+// limit (kWaitLimitNs) and flags ST_TIMEOUT_TMA, as a stalled pipeline would,
+// and the kernel returns normally.
+__global__ void stalled_wait_kernel(uint32_t* status) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int never_raised;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  never_raised = 0;
+  fence_barrier_init();
+  if (!mbar_wait(&bar, 0, &never_raised)) set_status(status, ST_TIMEOUT_TMA);
+}
+
+void launch_stalled_wait(uint32_t* status, cudaStream_t s) {
+  PARD_LAUNCH(stalled_wait_kernel, 1, 32, 0, s, false, status);
+}
+
 void launch_embed(const EmbedArgs& a, int grid, cudaStream_t s, bool pdl) {
   PARD_LAUNCH(embed_kernel, grid, 128, 0, s, pdl, a);
 }

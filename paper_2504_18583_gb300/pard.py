@@ -62,6 +62,7 @@ def lib() -> ctypes.CDLL:
         L.pard_draft.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp]
         L.pard_draft_sequential.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp]
         L.pard_set_mask_ids.argtypes = [vp, vp, i32, vp]
+        L.pard_selftest_stalled_wait.argtypes = [vp, vp]
         L.pard_verify.argtypes = [vp, vp, f32, vp, vp]
         L.pard_accept_commit.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp, vp, vp]
         L.pard_set_logits.argtypes = [vp, vp, vp, vp, f32, vp]
@@ -83,7 +84,7 @@ def lib() -> ctypes.CDLL:
         L.pard_fused_pass_used.argtypes = [vp]
         L.pard_fused_pass_used.restype = i32
         for name in ("pard_load_weights", "pard_prefill", "pard_draft", "pard_draft_sequential", "pard_verify",
-                     "pard_accept_commit", "pard_set_mask_ids",
+                     "pard_accept_commit", "pard_set_mask_ids", "pard_selftest_stalled_wait",
                      "pard_set_logits", "pard_get_state", "pard_read_kv", "pard_last_status"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
@@ -268,6 +269,10 @@ class PardEngine:
         _check(lib().pard_read_kv(self.ctx, model, layer, b, ctypes.cast(pos, ctypes.c_void_p), n, k.data_ptr(),
                                   v.data_ptr(), self.stream.cuda_stream), "pard_read_kv")
         return k, v
+
+    def selftest_stalled_wait(self):
+        """Enqueue the bounded-wait self test (its wait runs out after 2 s)."""
+        _check(lib().pard_selftest_stalled_wait(self.ctx, self.stream.cuda_stream), "pard_selftest_stalled_wait")
 
     def last_status(self) -> int:
         flags = ctypes.c_uint32(0)

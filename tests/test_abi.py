@@ -67,6 +67,7 @@ def test_load_rejects_bad_shapes_before_touching_the_device():
     assert code == -1
     assert pard.lib().pard_draft_sequential(None, 0, 1.0, 0, 0, None, None, None) == -1
     assert pard.lib().pard_set_mask_ids(None, None, 0, None) == -1
+    assert pard.lib().pard_selftest_stalled_wait(None, None) == -1
     assert pard.lib().pard_set_fused_pass(None, 1) == -1
     assert pard.lib().pard_fused_pass_used(None) == 0
 

@@ -95,6 +95,22 @@ def test_distinct_mask_ids_and_k12_match_oracle_every_step():
     P.eng.set_mask_ids(None)
 
 
+def test_stalled_wait_is_reported_and_the_context_stays_usable():
+    """Failure detection without a GPU fault: a kernel's bounded pipeline wait
+    on a barrier nothing completes gives up after its limit, sets the timeout
+    bit and returns; pard_last_status reports it, and the next decode steps
+    still match the oracle."""
+    wl = S.WORKLOADS["tiny"].replace(n_new=12)
+    P = Pair(wl)
+    P.prefill()
+    greedy_step(P, 1)
+    assert P.eng.last_status() == 0
+    P.eng.selftest_stalled_wait()
+    assert P.eng.last_status() == 1  # ST_TIMEOUT_TMA
+    greedy_step(P, 2)
+    assert P.eng.last_status() == 0
+
+
 def test_tiny_greedy_jittered_norms_batch_ragged():
     """Batch of 3 with prompts 17 / 33 / 50 tokens (page boundaries at
     several offsets), norm gains != 1, prefill chunks of 64 rows."""
