@@ -307,6 +307,81 @@ def test_distinct_mask_ids_keep_pard_lossless_and_reach_the_draft(tiny):
     assert np.array_equal(z_shared[0, 0], z[0, 0]) and not np.array_equal(z_shared[0, 1:], z[0, 1:])
 
 
+# --------------------------------------------------------------------------
+# COD data construction (Section 3.2, appendix algorithm and worked example)
+# --------------------------------------------------------------------------
+def test_cod_worked_example_from_the_paper():
+    """The appendix example: "tell me a story about", K = 3, r = 0.5.  With
+    m_{0,1} and m_{0,2} kept at +2 (the example's choice), the +3 candidates
+    are exactly {m_{1,2}, m_{1,3}} (m_{1,1} lost its prefix m_{0,0}) and one
+    of them is kept; m_{1,3} predicts "about" from [tell, me, m_{0,2}] and
+    m_{1,2} predicts "story" from [tell, m_{0,1}]."""
+    from oracle import cod
+    tell, me, a, story, about = 10, 11, 12, 13, 14
+    N = 4
+    assert cod.retained_count(N, 1, 0.5, 0.0) == 4
+    assert cod.retained_count(N, 2, 0.5, 0.0) == 2
+    assert cod.retained_count(N, 3, 0.5, 0.0) == 1
+    keep, counts = cod.cod_select(N, 3, 0.5, 0.0, seed=1, sample_id=0, forced=[[1, 2]])
+    assert cod.candidates(keep, 3, N) == [2, 3]
+    assert counts[:2] == [4, 2] and counts[2] == 1 and keep[1].sum() == 1 and keep[1, 2] + keep[1, 3] == 1
+    for pick, label, real in ((3, about, [tell, me]), (2, story, [tell])):
+        keep, _ = cod.cod_select(N, 3, 0.5, 0.0, seed=1, sample_id=0, forced=[[1, 2], [pick]])
+        rows = cod.packed_rows([tell, me, a, story, about], keep, [900, 901])
+        k3 = [row for row in rows if row[0] == 3][0]
+        assert k3[1] == 901 and k3[2] == pick and k3[3] == label and k3[5] == len(real)
+        pred = rows[k3[4]]
+        assert pred[0] == 2 and pred[1] == 900 and pred[2] == pick - 1
+        assert [rows[i][1] for i in range(k3[5])] == real
+
+
+def test_cod_counts_follow_the_geometric_retention():
+    """N_k = N max(r^(k-1), r_min) per subtask (Section 3.2); with r_min = 0
+    the total is N (1 - r^K) / (1 - r) up to the per-subtask rounding."""
+    from oracle import cod
+    N, K = 1000, 6
+    for r, r_min in ((0.5, 0.0), (0.7, 0.0), (0.5, 0.2)):
+        _, counts = cod.cod_select(N, K, r, r_min, seed=5, sample_id=3)
+        for k in range(1, K + 1):
+            assert counts[k - 1] == int(np.floor(N * max(r ** (k - 1), r_min) + 0.5)), (r, r_min, k)
+        if r_min == 0.0:
+            assert abs(sum(counts) - N * (1 - r ** K) / (1 - r)) <= K
+
+
+def test_cod_every_kept_row_has_its_whole_context():
+    """Integrity of prefix key-value states: every kept row of subtask k >= 3
+    has its predecessor chain down to subtask 2 kept; r = 1 keeps every row
+    (plain mask-token training)."""
+    from oracle import cod
+    rng = np.random.default_rng(7)
+    for t in range(30):
+        N, K = int(rng.integers(1, 60)), int(rng.integers(2, 9))
+        r, r_min = float(rng.uniform(0.2, 1.0)), float(rng.uniform(0.0, 0.3))
+        keep, counts = cod.cod_select(N, K, r, r_min, seed=t, sample_id=t)
+        for k in range(3, K + 1):
+            for j in range(N):
+                if keep[k - 2, j]:
+                    assert j >= k - 2 and all(keep[kk - 2, j - (k - kk)] for kk in range(2, k))
+        assert counts == [N] + [int(keep[k - 2].sum()) for k in range(2, K + 1)]
+    keep, _ = cod.cod_select(20, 5, 1.0, 0.0, seed=1, sample_id=1)
+    for k in range(2, 6):
+        assert keep[k - 2].tolist() == [0] * (k - 2) + [1] * (20 - k + 2)
+
+
+def test_cod_choice_is_uniform_over_candidates():
+    """The random choice of subtask 2 keeps each position with probability
+    n / N: chi-square over 400 samples, N = 10, n = 5."""
+    from oracle import cod
+    hits = np.zeros(10)
+    S_ = 400
+    for sid in range(S_):
+        keep, _ = cod.cod_select(10, 2, 0.5, 0.0, seed=11, sample_id=sid)
+        hits += keep[0]
+    exp = S_ * 0.5
+    chi2 = float((((hits - exp) ** 2) / exp).sum())
+    assert chi2 < 27.9  # 9 degrees of freedom, p = 0.001
+
+
 def test_greedy_accept_rule_every_length():
     rng = np.random.default_rng(3)
     K, V = 5, 11
