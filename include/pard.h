@@ -199,6 +199,23 @@ pard_status pard_read_kv(pard_ctx* ctx, int32_t model, int32_t layer, int32_t b,
  * PARD_ERR_DEVICE_CHECK when bits are set. */
 pard_status pard_last_status(pard_ctx* ctx, uint32_t* h_flags, void* stream);
 
+/* COD data construction (Section 3.2, appendix algorithm) for one training
+ * sample of n+1 tokens and K subtasks: d_keep[(k-2)*n + j] = 1 when row j of
+ * mask subtask k (k = 2..K; position j, fed mask m_{k-2}, labelled x_{j+1})
+ * is kept, and d_counts[k-1] = rows kept by subtask k (d_counts[0] = n:
+ * subtask 1, ordinary next-token training, keeps every row).  Subtask k keeps
+ * round(n * max(r^(k-1), r_min)) rows (r^(k-1) by repeated multiplication in
+ * double, half up), chosen among the rows whose predecessor (row j-1 of
+ * subtask k-1) is kept -- the integrity of prefix key-value states; every
+ * subtask-2 row qualifies, rows j < k-2 never do.  The choice keeps the
+ * candidates with the smallest Philox words (stream 3, step = sample_id,
+ * row k, v = j; ties to the lower j), so it is reproducible.  Bounds:
+ * 1 <= n <= 4096, 1 <= K <= 64, 0 < r <= 1, 0 <= r_min <= 1; d_keep holds
+ * (K-1)*n int32 (may be NULL when K = 1), d_counts K int32, both device
+ * memory.  Needs no context; enqueues one kernel on `stream`. */
+pard_status pard_cod_select(int32_t n, int32_t K, double r, double r_min, uint64_t seed, uint64_t sample_id,
+                            int32_t* d_keep, int32_t* d_counts, void* stream);
+
 /* Failure-path self test: enqueue one kernel whose bounded pipeline wait
  * (the one every GEMM stage uses) waits on a barrier nothing completes; after
  * the wait limit (2 s) it sets the timeout bit of the device status word

@@ -1172,6 +1172,20 @@ pard_status pard_last_status(pard_ctx* c, uint32_t* h_flags, void* stream) {
   });
 }
 
+pard_status pard_cod_select(int32_t n, int32_t K, double r, double r_min, uint64_t seed, uint64_t sample_id,
+                            int32_t* d_keep, int32_t* d_counts, void* stream) {
+  if (n < 1 || n > kCodMaxN) return fail(PARD_ERR_ARG, "COD sample rows outside [1, 4096]");
+  if (K < 1 || K > 64) return fail(PARD_ERR_ARG, "COD subtask count outside [1, 64]");
+  if (!(r > 0.0 && r <= 1.0) || !(r_min >= 0.0 && r_min <= 1.0))
+    return fail(PARD_ERR_ARG, "COD retention r outside (0, 1] or r_min outside [0, 1]");
+  if (!d_counts || (K > 1 && !d_keep)) return fail(PARD_ERR_ARG, "null output");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return guarded([&]() -> pard_status {
+    launch_cod(n, K, r, r_min, seed, sample_id, d_keep, d_counts, s);
+    return PARD_OK;
+  });
+}
+
 pard_status pard_selftest_stalled_wait(pard_ctx* c, void* stream) {
   if (!c) return fail(PARD_ERR_ARG, "null context");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

@@ -231,6 +231,9 @@ void launch_read_kv(const __nv_bfloat16* kc, const __nv_bfloat16* vc, const int*
                     int hkv, int hd, int page_size, __nv_bfloat16* ok, __nv_bfloat16* ov, cudaStream_t s);
 
 void launch_stalled_wait(uint32_t* status, cudaStream_t s);
+constexpr int kCodMaxN = 4096;  // rows per subtask of one COD sample
+void launch_cod(int N, int K, double r, double r_min, uint64_t seed, uint64_t sample_id, int32_t* keep,
+                int32_t* counts, cudaStream_t s);
 void launch_gemm(const GemmArgs& a, int tt, int grid, cudaStream_t s, bool pdl);
 int gemm_smem_bytes(int tt);
 void launch_attention(const AttnArgs& a, int grid_x, cudaStream_t s, bool pdl);

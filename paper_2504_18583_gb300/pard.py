@@ -63,6 +63,7 @@ def lib() -> ctypes.CDLL:
         L.pard_draft_sequential.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp]
         L.pard_set_mask_ids.argtypes = [vp, vp, i32, vp]
         L.pard_selftest_stalled_wait.argtypes = [vp, vp]
+        L.pard_cod_select.argtypes = [i32, i32, ctypes.c_double, ctypes.c_double, u64, u64, vp, vp, vp]
         L.pard_verify.argtypes = [vp, vp, f32, vp, vp]
         L.pard_accept_commit.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp, vp, vp]
         L.pard_set_logits.argtypes = [vp, vp, vp, vp, f32, vp]
@@ -84,11 +85,23 @@ def lib() -> ctypes.CDLL:
         L.pard_fused_pass_used.argtypes = [vp]
         L.pard_fused_pass_used.restype = i32
         for name in ("pard_load_weights", "pard_prefill", "pard_draft", "pard_draft_sequential", "pard_verify",
-                     "pard_accept_commit", "pard_set_mask_ids", "pard_selftest_stalled_wait",
+                     "pard_accept_commit", "pard_set_mask_ids", "pard_selftest_stalled_wait", "pard_cod_select",
                      "pard_set_logits", "pard_get_state", "pard_read_kv", "pard_last_status"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
+
+
+def cod_select(n: int, K: int, r: float, r_min: float, seed: int, sample_id: int, stream=None):
+    """COD data construction for one sample (pard_cod_select): returns device
+    tensors keep [K-1, n] and counts [K] (int32), enqueued on `stream`."""
+    import torch
+    keep = torch.zeros((max(K - 1, 1), n), dtype=torch.int32, device="cuda")
+    counts = torch.zeros(K, dtype=torch.int32, device="cuda")
+    s = stream if stream is not None else torch.cuda.current_stream()
+    _check(lib().pard_cod_select(n, K, float(r), float(r_min), seed, sample_id, keep.data_ptr(), counts.data_ptr(),
+                                 s.cuda_stream), "pard_cod_select")
+    return keep[:K - 1], counts
 
 
 class PardError(RuntimeError):

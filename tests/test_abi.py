@@ -68,6 +68,10 @@ def test_load_rejects_bad_shapes_before_touching_the_device():
     assert pard.lib().pard_draft_sequential(None, 0, 1.0, 0, 0, None, None, None) == -1
     assert pard.lib().pard_set_mask_ids(None, None, 0, None) == -1
     assert pard.lib().pard_selftest_stalled_wait(None, None) == -1
+    # COD: argument checks happen on the host, before any launch
+    for n, K, r, r_min in ((0, 3, 0.5, 0.0), (4097, 3, 0.5, 0.0), (10, 0, 0.5, 0.0), (10, 3, 0.0, 0.0),
+                           (10, 3, 1.5, 0.0), (10, 3, 0.5, -0.1)):
+        assert pard.lib().pard_cod_select(n, K, r, r_min, 0, 0, None, None, None) == -1
     assert pard.lib().pard_set_fused_pass(None, 1) == -1
     assert pard.lib().pard_fused_pass_used(None) == 0
 

@@ -111,6 +111,33 @@ def test_stalled_wait_is_reported_and_the_context_stays_usable():
     assert P.eng.last_status() == 0
 
 
+def test_cod_keep_flags_match_the_oracle_bit_exactly():
+    """COD data construction (Section 3.2, appendix algorithm) on the GPU:
+    keep flags and per-subtask counts identical to the oracle's for ragged
+    sample lengths, K = 1..8, several retention settings, the 4096-row
+    maximum and the degenerate cases (n = 1, r = 1, r_min = 1)."""
+    import torch
+    from oracle import cod
+    from paper_2504_18583_gb300 import pard
+    cases = [(1, 3, 0.5, 0.0), (4, 3, 0.5, 0.0), (37, 2, 0.5, 0.0), (500, 8, 0.5, 0.0), (777, 6, 0.7, 0.1),
+             (2048, 8, 0.5, 0.05), (4096, 8, 0.6, 0.0), (64, 1, 0.5, 0.0), (100, 5, 1.0, 0.0), (100, 5, 0.3, 1.0)]
+    for t, (n, K, r, r_min) in enumerate(cases):
+        keep_g, counts_g = pard.cod_select(n, K, r, r_min, seed=1000 + t, sample_id=t)
+        keep_o, counts_o = cod.cod_select(n, K, r, r_min, seed=1000 + t, sample_id=t)
+        torch.cuda.synchronize()
+        assert counts_g.cpu().tolist() == counts_o, (n, K, r, r_min)
+        assert np.array_equal(keep_g.cpu().numpy(), keep_o), (n, K, r, r_min)
+    # one 2048-row, K = 8 sample, timed on the device
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    pard.cod_select(2048, 8, 0.5, 0.0, 1, 0)
+    ev[0].record()
+    for i in range(20):
+        pard.cod_select(2048, 8, 0.5, 0.0, 1, i)
+    ev[1].record()
+    torch.cuda.synchronize()
+    print("COD 2048 rows, K = 8: %.1f us per sample" % (ev[0].elapsed_time(ev[1]) * 1e3 / 20))
+
+
 def test_tiny_greedy_jittered_norms_batch_ragged():
     """Batch of 3 with prompts 17 / 33 / 50 tokens (page boundaries at
     several offsets), norm gains != 1, prefill chunks of 64 rows."""
