@@ -16,6 +16,13 @@ oracle is timed on the host cores on a bounded sample (``cpu_baseline``).
 ``--impl reference`` times the CPU oracle itself, step for step.
 Under torchrun each rank runs an independent replica (the batch-1 step does
 not shard without tensor parallelism): value = all ranks' tokens / max time.
+
+The headline run also reports, on the same kernels: a planted-acceptance run
+(the verify input is the target's own continuation, corrupted at rate
+1 - alpha), the autoregressive baseline (K = 0) and vanilla speculative
+decoding (K sequential draft passes).  ``--workload`` picks the sampling or
+batch-16 workload, ``--batch`` overrides the batch (sweep), ``--layers`` and
+``--no-extras`` / ``--no-e2e`` / ``--no-cpu-baseline`` shorten profiling runs.
 """
 from __future__ import annotations
 
