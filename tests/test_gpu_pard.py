@@ -138,6 +138,32 @@ def test_cod_keep_flags_match_the_oracle_bit_exactly():
     print("COD 2048 rows, K = 8: %.1f us per sample" % (ev[0].elapsed_time(ev[1]) * 1e3 / 20))
 
 
+def test_page_pool_exhaustion_and_device_bounds_flag():
+    """Host and device checks without a fault: a batch whose page reservation
+    exceeds the pool returns PARD_ERR_NO_PAGES before any launch; a verify
+    candidate outside the vocabulary is caught by the row-plan kernel, which
+    flags ST_BAD_TOKEN (read by pard_last_status as PARD_ERR_DEVICE_CHECK)
+    and embeds token 0 instead of reading out of bounds."""
+    import torch
+    from paper_2504_18583_gb300 import pard
+    wl = S.WORKLOADS["tiny"].replace(n_new=20, prompt_len=40)
+    tw = S.device_weights(wl.target, wl.seed, S.TARGET)
+    dw = S.device_weights(wl.draft, wl.seed, S.DRAFT)
+    eng = pard.PardEngine(wl.target, tw, wl.draft, dw, max_batch=1, max_k=wl.K, max_ctx=256, n_pages=2,
+                          prefill_chunk=64)
+    with pytest.raises(pard.PardError) as e:
+        eng.prefill([list(range(1, 41))], wl.n_new, wl.K)
+    assert e.value.code == -3  # PARD_ERR_NO_PAGES: 40 + 20 + 2K positions need 5 pages of 16
+    P = Pair(wl)
+    P.prefill()
+    out = P.eng.alloc_step_outputs()
+    P.eng.draft(out)
+    bad = torch.full((1, wl.K), wl.target.vocab + 5, dtype=torch.int32, device="cuda")
+    P.eng.verify(out, bad)
+    assert P.eng.last_status() == 1 << 3  # ST_BAD_TOKEN
+    assert P.eng.last_status() == 0       # the word is cleared once read
+
+
 def test_tiny_greedy_jittered_norms_batch_ragged():
     """Batch of 3 with prompts 17 / 33 / 50 tokens (page boundaries at
     several offsets), norm gains != 1, prefill chunks of 64 rows."""

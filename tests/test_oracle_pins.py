@@ -382,6 +382,24 @@ def test_cod_choice_is_uniform_over_candidates():
     assert chi2 < 27.9  # 9 degrees of freedom, p = 0.001
 
 
+def test_rollback_then_recompute_gives_identical_cache_values(tiny):
+    """Rollback is by length only: after rows at positions p..p+2 are written
+    and the last is rejected, feeding another token at p+2 and then the
+    original one again rewrites exactly the first values (rows do not depend
+    on what was written past them)."""
+    wl, tw, _ = tiny
+    pr = wl.prompts()[0].tolist()
+    P0 = len(pr)
+    m = P.OracleModel(wl.target, tw, 1, 64)
+    m.forward(0, pr, range(P0), [])
+    m.forward(0, [5, 77, 300], [P0, P0 + 1, P0 + 2], [])
+    k1, v1 = m.kc[0][:, :P0 + 3].copy(), m.vc[0][:, :P0 + 3].copy()
+    m.forward(0, [1999], [P0 + 2], [])
+    assert not np.array_equal(m.kc[0][:, P0 + 2], k1[:, P0 + 2])
+    m.forward(0, [300], [P0 + 2], [])
+    assert np.array_equal(m.kc[0][:, :P0 + 3], k1) and np.array_equal(m.vc[0][:, :P0 + 3], v1)
+
+
 def test_greedy_accept_rule_every_length():
     rng = np.random.default_rng(3)
     K, V = 5, 11
