@@ -311,28 +311,39 @@ def test_distinct_mask_ids_keep_pard_lossless_and_reach_the_draft(tiny):
 # COD data construction (Section 3.2, appendix algorithm and worked example)
 # --------------------------------------------------------------------------
 def test_cod_worked_example_from_the_paper():
-    """The appendix example: "tell me a story about", K = 3, r = 0.5.  With
-    m_{0,1} and m_{0,2} kept at +2 (the example's choice), the +3 candidates
-    are exactly {m_{1,2}, m_{1,3}} (m_{1,1} lost its prefix m_{0,0}) and one
-    of them is kept; m_{1,3} predicts "about" from [tell, me, m_{0,2}] and
-    m_{1,2} predicts "story" from [tell, m_{0,1}]."""
+    """The appendix example (tests/golden/cod_worked_example.txt): with the
+    example's choice at +2, the +3 candidates, the number kept and the
+    contexts and labels of m_{1,2} and m_{1,3} are the ones the paper states."""
     from oracle import cod
-    tell, me, a, story, about = 10, 11, 12, 13, 14
-    N = 4
-    assert cod.retained_count(N, 1, 0.5, 0.0) == 4
-    assert cod.retained_count(N, 2, 0.5, 0.0) == 2
-    assert cod.retained_count(N, 3, 0.5, 0.0) == 1
-    keep, counts = cod.cod_select(N, 3, 0.5, 0.0, seed=1, sample_id=0, forced=[[1, 2]])
-    assert cod.candidates(keep, 3, N) == [2, 3]
-    assert counts[:2] == [4, 2] and counts[2] == 1 and keep[1].sum() == 1 and keep[1, 2] + keep[1, 3] == 1
-    for pick, label, real in ((3, about, [tell, me]), (2, story, [tell])):
-        keep, _ = cod.cod_select(N, 3, 0.5, 0.0, seed=1, sample_id=0, forced=[[1, 2], [pick]])
-        rows = cod.packed_rows([tell, me, a, story, about], keep, [900, 901])
+    g = {}
+    for line in open(os.path.join(GOLDEN, "cod_worked_example.txt")):
+        if line.strip() and not line.startswith("#"):
+            key, *vals = line.split()
+            g[key] = vals
+    words = g["tokens"]
+    ids = {w: 10 + i for i, w in enumerate(words)}
+    toks = [ids[w] for w in words]
+    N, K, r = len(toks) - 1, int(g["K"][0]), float(g["r"][0])
+    masks = [900, 901]
+    mask_name = {900: "m0", 901: "m1"}
+    kept_2 = [int(x) for x in g["kept_2"]]
+    assert cod.retained_count(N, 2, r, 0.0) == len(kept_2)
+    assert cod.retained_count(N, 3, r, 0.0) == int(g["n_kept_3"][0])
+    keep, counts = cod.cod_select(N, K, r, 0.0, seed=1, sample_id=0, forced=[kept_2])
+    assert cod.candidates(keep, 3, N) == [int(x) for x in g["candidates_3"]]
+    assert counts == [N, len(kept_2), int(g["n_kept_3"][0])]
+    for j in (int(x) for x in g["candidates_3"]):
+        keep, _ = cod.cod_select(N, K, r, 0.0, seed=1, sample_id=0, forced=[kept_2, [j]])
+        rows = cod.packed_rows(toks, keep, masks)
         k3 = [row for row in rows if row[0] == 3][0]
-        assert k3[1] == 901 and k3[2] == pick and k3[3] == label and k3[5] == len(real)
-        pred = rows[k3[4]]
-        assert pred[0] == 2 and pred[1] == 900 and pred[2] == pick - 1
-        assert [rows[i][1] for i in range(k3[5])] == real
+        real_words = [words[toks.index(rows[i][1])] for i in range(k3[5])]
+        chain, at = [], k3[4]
+        while at >= 0:
+            chain.append("%s%d" % (mask_name[rows[at][1]], rows[at][2]))
+            at = rows[at][4]
+        ctx = " ".join(real_words) + " | " + " ".join(reversed(chain))
+        assert ctx == " ".join(g["context_m1%d" % j]), (ctx, j)
+        assert words[toks.index(k3[3])] == g["label_m1%d" % j][0]
 
 
 def test_cod_counts_follow_the_geometric_retention():
