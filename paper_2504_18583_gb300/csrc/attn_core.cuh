@@ -235,7 +235,7 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
   int* spg = reinterpret_cast<int*>(smem + C::kPageOff);
   const bool cached = a.pt_ld <= kAttnPageCache;
 
-  // ---- round 1: row positions, the sequence's first position, page table row ----
+  // ---- first wave of loads: row positions, the sequence's first position, page table row ----
   const int pos_v = tid < nrows ? __ldcg(a.row_pos + row0 + tid) : -1;
   const int first_v = (tid == 0 && nrows > 0) ? __ldcg(a.row_pos + s0) : 0;
   int pg_v[kAttnPageCache / kAttnThreads];
@@ -272,7 +272,7 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
   }
   wait_q();
 
-  // ---- round 2: Q ----
+  // ---- second wave of loads: Q ----
   // q is rewritten by every layer, by other CTAs of a persistent grid: L2 loads
   constexpr int kQIter = kMaxQV * (HD / 4) / kAttnThreads;  // 8 or 16 float4 per thread
   constexpr int kQGroup = kQIter < 8 ? kQIter : 8;
