@@ -722,7 +722,7 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
     int major = 0, minor = 0;
     CK(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev));
     CK(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev));
-    if (major != 10) return fail(PARD_ERR_CUDA, "this build runs on compute capability 10.x (GB300, sm_103a) only");
+    if (major != 10) return fail(PARD_ERR_CUDA, "libpard is compiled for compute capability 10.x (GB300, sm_103a) only");
     c->sm = std::min(c->sm, 160);
     c->lim = *lim;
     c->D = make_dims(*tcfg, *dcfg, *lim, c->sm);
