@@ -7,6 +7,7 @@ or header is newer than the library.
 from __future__ import annotations
 
 import concurrent.futures as cf
+import fcntl
 import glob
 import os
 import shutil
@@ -51,10 +52,23 @@ def up_to_date() -> bool:
 
 
 def build(verbose: bool = False, extra_flags=()) -> str:
-    """Compile every .cu under csrc/ and link libpard.so; returns its path."""
+    """Compile every .cu under csrc/ and link libpard.so; returns its path.
+    Processes that build at once (one per rank under torch.distributed.run)
+    take a file lock, so one compiles and the others find it up to date."""
     if up_to_date() and not extra_flags:
         return LIB
     os.makedirs(BUILD, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            if up_to_date() and not extra_flags:
+                return LIB
+            return _compile_and_link(verbose, extra_flags)
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
+def _compile_and_link(verbose: bool, extra_flags) -> str:
     cc = nvcc()
 
     def compile_one(src):
