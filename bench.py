@@ -71,11 +71,11 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def measured_verify_traffic(persistent: bool):
+def measured_verify_traffic():
     """DRAM bytes of one verify pass from the committed ncu summary, or None when
-    the kernels changed since it was taken (or the pass runs another kernel)."""
+    the kernels changed since it was taken."""
     p = os.path.join(ROOT, "profiles", "verify_pass_dram_traffic_8b.json")
-    if persistent or not os.path.exists(p):
+    if not os.path.exists(p):
         return None
     d = json.load(open(p))
     return d["verify_traffic_bytes"] if d.get("csrc_sha") == kernel_source_hash() else None
@@ -254,8 +254,6 @@ def main():
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the planted-acceptance and autoregressive runs (profiling runs: the timed steps "
                          "are then the last launches)")
-    ap.add_argument("--persistent", action="store_true",
-                    help="run draft / verify as one persistent kernel instead of one kernel per phase")
     ap.add_argument("--workload", default="8b_greedy", choices=["8b_greedy", "8b_sample", "8b_batch16"],
                     help="8b_greedy (the headline), 8b_sample (T = 1, K = 6), 8b_batch16 (16 ragged prompts, K = 6)")
     ap.add_argument("--layers", type=int, default=0,
@@ -298,7 +296,6 @@ def main():
     eng = pard.PardEngine(wl.target, tw, wl.draft, dw, max_batch=wl.batch, max_k=wl.K, max_ctx=max_ctx,
                           n_pages=wl.n_pages(), prefill_chunk=512, page_order_target=wl.page_order(S.TARGET),
                           page_order_draft=wl.page_order(S.DRAFT))
-    eng.set_fused_pass(args.persistent)
     stream = eng.stream
 
     sample, temp, seed = wl.sample, wl.temperature, 1
@@ -353,7 +350,6 @@ def main():
     clk = clocks.stop()
     n_state = eng.state()[0][0]
     flags = eng.last_status()
-    fused_used = eng.fused_pass_used()
 
     # max over ranks
     ms_max, tot_toks = aggregate_over_ranks(ms, toks, ws)
@@ -528,14 +524,12 @@ def main():
                                 + (f" (batch overridden to {wl.batch})" if args.batch else "")),
                    "batch": wl.batch, "parallelism": f"replicas{ws}",
                    "l2": "inputs larger than L2: 17.5 GB of weights stream from HBM every step",
-                   "acceptance": "random-init draft: ~0 candidates accepted, ~1 token per step",
-                   "forward_pass": "persistent" if fused_used else "per_phase"},
+                   "acceptance": "random-init draft: ~0 candidates accepted, ~1 token per step"},
         "roofline": {"bound": "hbm",
-                     "kernel": ("verify pass: embedding kernel + one persistent fwd_kernel launch" if fused_used
-                                else "verify pass (all its launches; GEMM-dominated)"),
+                     "kernel": "verify pass (all its launches; GEMM-dominated)",
                      "achieved": ver_gbs, "peak": peak, "unit": "GB/s", "frac": ver_gbs / peak,
                      "peak_kind": peak_kind,
-                     "traffic": (measured_verify_traffic(fused_used)
+                     "traffic": (measured_verify_traffic()
                                  if args.workload == "8b_greedy" and not args.layers and not args.batch else None),
                      "traffic_source": "profiles/verify_pass_dram_traffic_8b.json (ncu DRAM bytes, 2-layer capture "
                                        "scaled to 32 layers; null if the kernels changed since)",

@@ -88,7 +88,14 @@ size_t pard_workspace_bytes(const pard_model_cfg* target, const pard_model_cfg* 
  * [layer][K|V][page][kv_head][token][head_dim].  Host only. */
 size_t pard_kv_pool_bytes(const pard_model_cfg* target, const pard_model_cfg* draft, const pard_limits* lim);
 
-/* Validate shapes, record the borrowed pointers, carve the workspace and
+/* Loads the two models of the method: the target model that verifies and the
+ * PARD draft model that proposes K tokens per forward pass (Section 3.1).
+ * Section 4.1 trains the smallest variant of a model series as the draft of
+ * that series' targets (e.g. the LLaMA3.1-8B and LLaMA3.3-70B rows of
+ * Table 1); both are Llama-style decoders with bf16 weights.  The caller owns
+ * the weights, the KV page pool and the workspace; the library borrows them
+ * until pard_destroy.
+ * Validate shapes, record the borrowed pointers, carve the workspace and
  * build TMA descriptors and RoPE tables.
  * IN-PLACE PACKING: every projection and LM-head matrix whose row count is a
  * multiple of 128 (64 for wg/wu) and whose column count is a multiple of 64
@@ -109,7 +116,11 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* target, cons
 
 /* Prefill both models on `batch` prompts (d_tokens: the prompts
  * concatenated, h_lens[b] tokens each) and emit each sequence's first new
- * token into d_first_token[b] (argmax, or a Gumbel-max draw at
+ * token into d_first_token[b].  This is the prompt pass that precedes the
+ * decode iterations of Section 2.2: it fills the target's and the draft's KV
+ * caches with the prompt (the prefix key-value states the draft and verify
+ * passes attend to) and the target's last-row logits give x_n, the first
+ * token that the first draft pass extends (argmax, or a Gumbel-max draw at
  * `temperature` with Philox stream 2, step 0 when sample != 0).
  * Reserves ceil((len + n_new + 2K) / page_size) pages per sequence and
  * model, in sequence order, from the front of the page order.
@@ -179,9 +190,22 @@ pard_status pard_accept_commit(pard_ctx* ctx, int32_t sample, float temperature,
 
 /* Replace the logits the next pard_accept_commit reads (testing the
  * acceptance rule on given inputs): d_target_logits [B][K+1][vocab],
- * d_draft_logits [B][K][vocab] (may be NULL when greedy), d_draft [B][K]. */
+ * d_draft_logits [B][K][vocab] (may be NULL when greedy), d_draft [B][K].
+ * A candidate outside [0, vocab) is rejected at its offset and flags
+ * ST_BAD_TOKEN in the device status word. */
 pard_status pard_set_logits(pard_ctx* ctx, const float* d_target_logits, const float* d_draft_logits,
                             const int32_t* d_draft, float temperature, void* stream);
+
+/* Candidates from given draft logits (testing the draft pass's token
+ * selection, Eq. 6, on identical inputs): d_draft_logits [B][K][vocab] take
+ * the place of the logits pard_draft reads at its K prediction rows;
+ * candidate d_i = argmax z_i, or (sample != 0) the Gumbel-max draw from
+ * softmax(z_i / temperature) with Philox stream 0, row i -- the selection
+ * pard_draft makes from its LM head's tile statistics.  The candidates, the
+ * logits and their row normalisers become the ones the next pard_verify /
+ * pard_accept_commit use.  Writes d_draft_out [B][K]. */
+pard_status pard_set_draft_logits(pard_ctx* ctx, const float* d_draft_logits, int32_t sample, float temperature,
+                                  uint64_t seed, uint64_t step, int32_t* d_draft_out, void* stream);
 
 /* Host copy of per-sequence state: h_n [B] (tokens so far, incl. pending),
  * h_generated [B], h_done [B].  Synchronises `stream`.  Any may be NULL. */
@@ -235,8 +259,9 @@ pard_status pard_unpack_weights(pard_ctx* ctx, void* stream);
  * same kernels, same results): d_target_logits [batch][K+1][vocab],
  * d_draft_logits [batch][K][vocab] (needed only when sample != 0), d_draft
  * [batch][K]; outputs d_accept_len [batch] and d_emitted [batch][K+1] (-1
- * after the emitted tokens).  Nothing is committed anywhere: no context is
- * involved.
+ * after the emitted tokens).  A candidate outside [0, vocab) is never read
+ * from the logits: it counts as a rejection at its offset.  Nothing is
+ * committed anywhere: no context is involved.
  * Scratch: one fixed file-scope device array of about 6.3 MiB, sized for
  * batch <= 16, 1 <= K <= 8, vocab <= 128256 (vocab a multiple of 8); larger
  * sizes return PARD_ERR_ARG with a message.  Every GPU that loads the
@@ -254,20 +279,22 @@ pard_status pard_accept_noalloc(const float* d_target_logits, const float* d_dra
 /* Kernel launches the last call enqueued (for launch accounting). */
 int32_t pard_launch_count(pard_ctx* ctx);
 
-/* Chooses how pard_draft / pard_verify run the forward pass (Sec. 3.1 draft
- * pass, Sec. 3.2 verify pass).  enable = 1: a pass of at most 16
- * rows (batch x 2K draft rows, batch x (K+1) verify rows) over fully packed
- * weights, head_dim 64 or 128 and 2, 4 or 8 query heads per KV head runs as one
- * persistent cooperative kernel (one CTA per SM) that streams every layer's
- * weights and the LM head back to back; other passes, and every pass when the
- * GPU cannot hold the cooperative grid, run one kernel per phase.  enable = 0
- * (the default): always one kernel per phase.  Both compute the same results up to the order
- * of floating-point sums.  Takes effect at the next pard_prefill.  Returns
- * PARD_ERR_ARG for a null context. */
-pard_status pard_set_fused_pass(pard_ctx* ctx, int32_t enable);
-
-/* 1 when the last pard_draft or pard_verify ran the persistent kernel, else 0. */
-int32_t pard_fused_pass_used(pard_ctx* ctx);
+/* Diagnostics of the attention kernel (Section 2.2: the verify pass attends
+ * over the full prefix; Eq. 6: so does the draft pass).  The key range of
+ * one (sequence, kv head, row block) unit is split over the CTAs of one
+ * thread-block cluster, whose partial results are combined either by a push
+ * into each finishing CTA's shared memory (when the receive area fits beside
+ * the CTAs' key/value buffers: short contexts) or by a pull over distributed
+ * shared memory (long contexts).  pard_attention_paths synchronises `stream`
+ * and returns in *h_bits which forms ran since the last read (bit 0: push,
+ * bit 1: pull, bit 3 + n: a cluster of n CTAs), then clears the record.
+ * pard_set_attention_split_cap limits the key splits of one unit to cap
+ * CTAs (1..16; 0 restores the default 16) from the next pass on: the
+ * launcher falls back to 8-CTA clusters on a GPU that cannot place 16, and a
+ * cap gives that form on any GPU.  Both return PARD_ERR_ARG for a null
+ * context or a cap outside [0, 16]. */
+pard_status pard_attention_paths(pard_ctx* ctx, uint32_t* h_bits, void* stream);
+pard_status pard_set_attention_split_cap(pard_ctx* ctx, int32_t cap);
 
 /* Thread-local message for the last failing call ("" if none). */
 const char* pard_last_error(void);

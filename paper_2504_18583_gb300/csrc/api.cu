@@ -95,7 +95,6 @@ struct Dims {
   int gcap;         // rows of the prefill LM-head input
   int dmax, qdmax, ffnmax, vocab, hkvmax, hdmax, w_tiles, pt_ld, sm;
   int ffn_pad;      // widest FFN rounded up to whole 64-column blocks
-  int fwd_phases;   // phase capacity of one persistent-pass table (5 per layer + LM head)
 };
 
 int round_up(int x, int m) { return (x + m - 1) / m * m; }
@@ -115,7 +114,6 @@ Dims make_dims(const pard_model_cfg& t, const pard_model_cfg& d, const pard_limi
   D.w_tiles = (t.vocab + kTileN - 1) / kTileN;
   D.pt_ld = (lim.max_ctx + lim.page_size - 1) / lim.page_size;
   D.sm = sm;
-  D.fwd_phases = 5 * std::max(t.n_layers, d.n_layers) + 1;
   return D;
 }
 
@@ -126,8 +124,7 @@ struct WsOffsets {
   size_t row_tok, row_pos, row_seq, row_out, row_gi, seq_row0, m_dev;
   size_t g_row_seq, g_row_gi, g_m;
   size_t st_n, st_pc, st_pend, st_gen, st_max, st_done, st_d, st_dnorm, st_sa, st_snorm, st_spart, st_scnt;
-  size_t call, status, tmp_pos, pt[2], rope[2], g_plen, pack_tmp, mask_ids;
-  size_t fwd_tab, fwd_done, fwd_apart, fwd_acnt;
+  size_t call, status, paths, tmp_pos, pt[2], rope[2], g_plen, pack_tmp, mask_ids;
   size_t total;
 };
 
@@ -175,18 +172,13 @@ WsOffsets layout_ws(const Dims& D, const pard_limits& lim) {
   o.st_scnt = L.take((size_t)B * 4);
   o.call = L.take(sizeof(CallArgs));
   o.status = L.take(4);
+  o.paths = L.take(4);
   o.tmp_pos = L.take(4096 * 4);
   for (int mi = 0; mi < 2; ++mi) o.pt[mi] = L.take((size_t)B * D.pt_ld * 4);
   for (int mi = 0; mi < 2; ++mi) o.rope[mi] = L.take((size_t)D.pt_ld * lim.page_size * (D.hdmax / 2) * 8);
   o.g_plen = L.take((size_t)B * 4);
   o.mask_ids = L.take((size_t)std::max(K, 1) * 4);
   o.pack_tmp = L.take(kPackTmpBytes);
-  // persistent pass: 4 phase tables ([model][logits kept]), their completion
-  // counters, and the attention split partials and arrival counters
-  o.fwd_tab = L.take((size_t)4 * D.fwd_phases * sizeof(Phase));
-  o.fwd_done = L.take((size_t)4 * D.fwd_phases * 4);
-  o.fwd_apart = L.take((size_t)kFwdMaxAttnItems * kMaxQVRows * (D.hdmax + 2) * 4);
-  o.fwd_acnt = L.take((size_t)kFwdMaxAttnItems * 4);
   o.total = L.total + 256;
   return o;
 }
@@ -279,6 +271,8 @@ struct pard_ctx {
   DevState st;
   CallArgs* call;
   uint32_t* status;
+  uint32_t* paths;        // attention combine paths taken since the last read
+  int attn_split_cap = kMaxAttnSplit;  // key splits per attention cluster, at most
   int* tmp_pos;
   int* g_plen;
   int* mask_ids;          // per-offset draft mask ids (used when n_mask_ids > 0)
@@ -292,20 +286,6 @@ struct pard_ctx {
   std::vector<std::pair<__nv_bfloat16*, int>> packed_list;  // (matrix, R) packed in place, with N, K below
   std::vector<std::pair<int, int>> packed_shape;
   int launches = 0;
-  // persistent pass, per [model][logits kept]: phase table in the workspace,
-  // its completion counters and how many passes it has run
-  struct FwdTable {
-    Phase* dev = nullptr;
-    unsigned* done = nullptr;
-    int n = 0;
-    unsigned passes = 0;
-    bool ok = false;
-  } fwd[2][2];
-  float* fwd_apart = nullptr;
-  int* fwd_acnt = nullptr;
-  bool fwd_enabled = false;  // persistent pass opt-in (pard_set_fused_pass)
-  bool fwd_used = false;  // the last draft / verify ran the persistent pass
-
   template <typename T>
   T* at(size_t off) { return reinterpret_cast<T*>(ws + off); }
 };
@@ -341,8 +321,9 @@ void run_gemm(pard_ctx* c, GemmArgs& a, int tt, cudaStream_t s) {
 }
 
 // Attention work decomposition of a pass: row blocks per sequence, groups
-// (sequence x kv head x row block) and key splits (<= 16, about two CTAs per
-// SM, at most one per 32-key chunk of the longest context).
+// (sequence x kv head x row block) and key splits (<= 16 or the context's
+// cap, about two CTAs per SM, at most one per 32-key chunk of the longest
+// context).
 struct AttnGeom {
   int row_blocks, groups, n_split;
 };
@@ -353,7 +334,7 @@ AttnGeom attn_geometry(pard_ctx* c, int mi, int rows_per_seq, int batch) {
   g.row_blocks = (rows_per_seq + rb_rows - 1) / rb_rows;
   g.groups = batch * cf.n_kv_heads * g.row_blocks;
   const int n_kt = (c->lim.max_ctx + 31) / 32;  // 32-key chunks at the longest context
-  g.n_split = std::max(1, std::min({16, n_kt, (2 * c->sm + g.groups - 1) / g.groups}));
+  g.n_split = std::max(1, std::min({c->attn_split_cap, n_kt, (2 * c->sm + g.groups - 1) / g.groups}));
   return g;
 }
 
@@ -408,6 +389,7 @@ LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch
     a.scale = (float)(1.0 / std::sqrt((double)cf.head_dim));
     a.x_out = c->xo; a.x_rows = 2 * c->D.MC;
     a.status = c->status;
+    a.paths = c->paths;
   }
   // O projection + residual; emits x = h * g_mlp and the new row sums of squares
   {
@@ -503,115 +485,6 @@ void run_lm_head(pard_ctx* c, int mi, const __nv_bfloat16* x, int x_rows, const 
   GemmArgs a = lm_args(c, mi, x, x_rows, ssq_in, rows_cap, tt, m_dev, logits, row_out, row_gi, row_seq, stats, stats_i,
                        gumbel_stream);
   run_gemm(c, a, tt, s);
-}
-
-// ---------------------------------------------------------------------------
-// Persistent pass: the phase table of one decode forward (draft or verify),
-// run by one cooperative launch of fwd_kernel instead of 5 launches per layer
-// plus the LM head.  It covers passes of <= 16 rows over fully packed weights
-// with head shapes the kernel is instantiated for; everything else (prefill,
-// larger batches) takes the per-phase kernels.
-// ---------------------------------------------------------------------------
-bool fwd_shape_ok(const Model& M) {
-  const int hd = M.cfg.head_dim, group = M.cfg.n_q_heads / M.cfg.n_kv_heads;
-  if (!((hd == 128 || hd == 64) && (group == 2 || group == 4 || group == 8))) return false;
-  if (!M.lm_pk) return false;
-  for (int l = 0; l < M.cfg.n_layers; ++l)
-    for (int w : {W_Q, W_K, W_V, W_O, W_G, W_U, W_D})
-      if (!M.P[l].t[w]) return false;
-  return true;
-}
-
-// Builds (on the host) and uploads the phase table of model mi for the
-// current batch and K.  keep: the LM head also writes full logits.
-void build_fwd(pard_ctx* c, int mi, int keep, cudaStream_t s) {
-  pard_ctx::FwdTable& T = c->fwd[mi][keep];
-  T.ok = false;
-  T.n = 0;
-  T.passes = 0;
-  Model& M = c->m[mi];
-  const bool draft = mi == 1;
-  const int rows_per_seq = draft ? 2 * c->K : c->K + 1;
-  const int rows_cap = c->batch * rows_per_seq;
-  if (!c->fwd_enabled || rows_cap == 0 || rows_cap > kFwdTT || !fwd_shape_ok(M)) return;
-  if (5 * M.cfg.n_layers + 1 > c->D.fwd_phases) return;
-  AttnGeom geo = attn_geometry(c, mi, rows_per_seq, c->batch);
-  // one CTA per SM runs the attention items (group, split) = c, c + grid, ...
-  const int n_kt = (c->lim.max_ctx + 63) / 64;
-  geo.n_split = std::max(1, std::min({kFwdMaxSplit, n_kt, c->sm / std::max(1, geo.groups)}));
-  if (geo.groups * geo.n_split > kFwdMaxAttnItems) return;
-  std::vector<Phase> ph;
-  ph.reserve(5 * M.cfg.n_layers + 1);
-  auto gemm_phase = [&](const GemmArgs& g, int dep) {
-    Phase p;
-    std::memset(&p, 0, sizeof(p));
-    p.type = PH_GEMM;
-    p.dep = dep;
-    p.g = g;
-    ph.push_back(p);
-  };
-  for (int l = 0; l < M.cfg.n_layers; ++l) {
-    LayerPlan P = layer_plan(c, mi, l, rows_cap, kFwdTT, c->batch, M.page_table, geo, draft ? 0 : c->K + 1);
-    const int prev = (int)ph.size() - 1;  // -1 for the first layer: the embedding kernel precedes the launch
-    gemm_phase(P.qkv, prev);
-    Phase a;
-    std::memset(&a, 0, sizeof(a));
-    a.type = PH_ATTN;
-    a.dep = (int)ph.size() - 1;
-    a.attn_groups = geo.groups;
-    a.attn_split = geo.n_split;
-    a.at = P.at;
-    ph.push_back(a);
-    gemm_phase(P.o, (int)ph.size() - 1);
-    gemm_phase(P.gu, (int)ph.size() - 1);
-    gemm_phase(P.dn, (int)ph.size() - 1);
-  }
-  GemmArgs lm = draft ? lm_args(c, 1, c->xd, 2 * c->D.MC, c->ssq, rows_cap, kFwdTT, c->rp.m_dev,
-                                keep ? c->dlogits : nullptr, c->rp.row_out, c->rp.row_gi, c->rp.row_seq, c->stats_d,
-                                c->stats_id, STREAM_DRAFT)
-                      : lm_args(c, 0, c->xd, 2 * c->D.MC, c->ssq, rows_cap, kFwdTT, c->rp.m_dev,
-                                keep ? c->logits : nullptr, c->rp.row_out, nullptr, c->rp.row_seq, c->stats_t,
-                                c->stats_it, STREAM_BONUS);
-  gemm_phase(lm, (int)ph.size() - 1);
-  for (const Phase& p : ph)
-    if (p.type == PH_GEMM && p.g.tok_tiles != 1) return;
-  CK(cudaMemcpyAsync(T.dev, ph.data(), ph.size() * sizeof(Phase), cudaMemcpyHostToDevice, s));
-  CK(cudaMemsetAsync(T.done, 0, ph.size() * 4, s));
-  CK(cudaStreamSynchronize(s));
-  T.n = (int)ph.size();
-  T.ok = true;
-}
-
-// Runs the persistent pass of model mi if its table is usable; false means
-// the caller runs the per-phase kernels instead.
-bool try_fwd(pard_ctx* c, int mi, int keep, cudaStream_t s) {
-  pard_ctx::FwdTable& T = c->fwd[mi][keep];
-  c->fwd_used = false;
-  if (!c->fwd_enabled || !T.ok) return false;
-  FwdArgs f;
-  std::memset(&f, 0, sizeof(f));
-  f.phases = T.dev;
-  f.n_phases = T.n;
-  f.done = T.done;
-  f.target = (T.passes + 1) * (unsigned)c->sm;
-  f.attn_part = c->fwd_apart;
-  f.attn_cnt = c->fwd_acnt;
-  f.status = c->status;
-  f.m_dev = c->rp.m_dev;
-  f.m_cap = c->D.MC;
-  const Model& M = c->m[mi];
-  cudaError_t e = launch_fwd(f, M.cfg.head_dim, M.cfg.n_q_heads / M.cfg.n_kv_heads, c->sm, s);
-  if (e != cudaSuccess) {
-    // not launchable here (e.g. the grid cannot be co-resident): per-phase kernels from now on
-    (void)cudaGetLastError();
-    for (auto& row : c->fwd)
-      for (auto& t : row) t.ok = false;
-    return false;
-  }
-  T.passes++;
-  c->launches++;
-  c->fwd_used = true;
-  return true;
 }
 
 EmbedArgs embed_base(pard_ctx* c, int mi, int mode) {
@@ -746,22 +619,15 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
     c->st.samp_norm = c->at<float4>(o.st_snorm); c->st.samp_part = c->at<float2>(o.st_spart);
     c->st.samp_cnt = c->at<int>(o.st_scnt); c->st.kmax = lim->max_k;
     c->call = c->at<CallArgs>(o.call); c->status = c->at<uint32_t>(o.status);
+    c->paths = c->at<uint32_t>(o.paths);
     c->tmp_pos = c->at<int>(o.tmp_pos); c->g_plen = c->at<int>(o.g_plen);
     c->mask_ids = c->at<int>(o.mask_ids);
-    for (int mi = 0; mi < 2; ++mi)
-      for (int kl = 0; kl < 2; ++kl) {
-        const size_t t = (size_t)(2 * mi + kl) * c->D.fwd_phases;
-        c->fwd[mi][kl].dev = c->at<Phase>(o.fwd_tab) + t;
-        c->fwd[mi][kl].done = c->at<unsigned>(o.fwd_done) + t;
-      }
-    c->fwd_apart = c->at<float>(o.fwd_apart);
-    c->fwd_acnt = c->at<int>(o.fwd_acnt);
 
     // counters start at zero; the reduction kernels leave them at zero
     CK(cudaMemsetAsync(c->gcnt, 0, 65536 * 4, s));
-    CK(cudaMemsetAsync(c->fwd_acnt, 0, (size_t)kFwdMaxAttnItems * 4, s));
     CK(cudaMemsetAsync(c->st.samp_cnt, 0, lim->max_batch * 4, s));
     CK(cudaMemsetAsync(c->status, 0, 4, s));
+    CK(cudaMemsetAsync(c->paths, 0, 4, s));
     CK(cudaMemsetAsync(c->xd, 0, (size_t)2 * c->D.MC * c->D.dmax * 2, s));
     CK(cudaMemsetAsync(c->xo, 0, (size_t)2 * c->D.MC * c->D.qdmax * 2, s));
     CK(cudaMemsetAsync(c->xf, 0, (size_t)2 * c->D.MC * c->D.ffn_pad * 2, s));
@@ -936,8 +802,6 @@ pard_status pard_prefill(pard_ctx* c, const int32_t* d_tokens, const int32_t* h_
     sa.out = d_first; sa.plen = c->g_plen; sa.n_new = n_new;
     launch_select(sa, s, true);
     c->launches++;
-    for (int mi = 0; mi < 2; ++mi)
-      for (int keep = 0; keep < 2; ++keep) build_fwd(c, mi, keep, s);
     CK(cudaStreamSynchronize(s));
     CK(cudaGetLastError());
     c->prefilled = true;
@@ -963,12 +827,10 @@ pard_status pard_draft(pard_ctx* c, int32_t sample, float temperature, uint64_t 
     c->launches++;
     Model& M = c->m[1];
     const int keep = (sample || d_logits) ? 1 : 0;
-    if (!try_fwd(c, 1, keep, s)) {
-      run_layers(c, 1, rows_cap, c->batch, 2 * c->K, M.page_table, s);
-      const int tt = pick_tt(rows_cap);
-      run_lm_head(c, 1, c->xd, 2 * c->D.MC, c->ssq, rows_cap, tt, c->rp.m_dev, keep ? c->dlogits : nullptr,
-                  c->rp.row_out, c->rp.row_gi, c->rp.row_seq, c->stats_d, c->stats_id, STREAM_DRAFT, s);
-    }
+    run_layers(c, 1, rows_cap, c->batch, 2 * c->K, M.page_table, s);
+    run_lm_head(c, 1, c->xd, 2 * c->D.MC, c->ssq, rows_cap, pick_tt(rows_cap), c->rp.m_dev,
+                keep ? c->dlogits : nullptr, c->rp.row_out, c->rp.row_gi, c->rp.row_seq, c->stats_d, c->stats_id,
+                STREAM_DRAFT, s);
     SelectArgs sa;
     std::memset(&sa, 0, sizeof(sa));
     sa.mode = SEL_DRAFT;
@@ -1050,12 +912,10 @@ pard_status pard_verify(pard_ctx* c, const int32_t* d_draft_in, float temperatur
     Model& M = c->m[0];
     // K = 0 (autoregressive) keeps its single row of logits for a sampled accept
     const int keep = (c->last_draft_sampled || d_logits_out || c->K == 0) ? 1 : 0;
-    if (!try_fwd(c, 0, keep, s)) {
-      run_layers(c, 0, rows_cap, c->batch, c->K + 1, M.page_table, s, c->K + 1);  // K + 1 rows per sequence
-      const int tt = pick_tt(rows_cap);
-      run_lm_head(c, 0, c->xd, 2 * c->D.MC, c->ssq, rows_cap, tt, c->rp.m_dev, keep ? c->logits : nullptr,
-                  c->rp.row_out, nullptr, c->rp.row_seq, c->stats_t, c->stats_it, STREAM_BONUS, s);
-    }
+    run_layers(c, 0, rows_cap, c->batch, c->K + 1, M.page_table, s, c->K + 1);  // K + 1 rows per sequence
+    run_lm_head(c, 0, c->xd, 2 * c->D.MC, c->ssq, rows_cap, pick_tt(rows_cap), c->rp.m_dev,
+                keep ? c->logits : nullptr, c->rp.row_out, nullptr, c->rp.row_seq, c->stats_t, c->stats_it,
+                STREAM_BONUS, s);
     if (d_logits_out)
       CK(cudaMemcpyAsync(d_logits_out, c->logits, (size_t)c->batch * (c->K + 1) * c->D.vocab * 4,
                          cudaMemcpyDeviceToDevice, s));
@@ -1080,6 +940,7 @@ pard_status pard_accept_commit(pard_ctx* c, int32_t sample, float temperature, u
     a.call = c->call; a.st = c->st;
     a.page_table = c->m[0].page_table; a.pt_ld = c->D.pt_ld; a.page_size = c->lim.page_size;
     a.accept_len = d_accept_len; a.emitted = d_emitted; a.kv_slots = d_kv_slots; a.n_emit = d_n_emit;
+    a.status = c->status;
     if (sample) {
       launch_accept_sample(a, s, true);
       c->launches += 2;
@@ -1103,11 +964,11 @@ pard_status pard_set_logits(pard_ctx* c, const float* y, const float* z, const i
     CK(cudaMemcpyAsync(c->logits, y, (size_t)B * (K + 1) * V * 4, cudaMemcpyDeviceToDevice, s));
     CK(cudaMemcpy2DAsync(c->st.d, c->st.kmax * 4, d, K * 4, K * 4, B, cudaMemcpyDeviceToDevice, s));
     set_call(c, 0, 0, temperature, 1, s);
-    launch_row_stats(c->logits, B * (K + 1), V, c->D.w_tiles, c->D.MC, c->call, c->stats_t, c->stats_it, s);
+    launch_row_stats(c->logits, B * (K + 1), V, c->D.w_tiles, c->D.MC, c->call, -1, 1, c->stats_t, c->stats_it, s);
     c->launches++;
     if (z) {
       CK(cudaMemcpyAsync(c->dlogits, z, (size_t)B * K * V * 4, cudaMemcpyDeviceToDevice, s));
-      launch_row_stats(c->dlogits, B * K, V, c->D.w_tiles, c->D.MC, c->call, c->stats_d, c->stats_id, s);
+      launch_row_stats(c->dlogits, B * K, V, c->D.w_tiles, c->D.MC, c->call, -1, 1, c->stats_d, c->stats_id, s);
       SelectArgs sa;
       std::memset(&sa, 0, sizeof(sa));
       sa.mode = SEL_NORM_ONLY;
@@ -1116,6 +977,32 @@ pard_status pard_set_logits(pard_ctx* c, const float* y, const float* z, const i
       launch_select(sa, s, false);
       c->launches += 2;
     }
+    return PARD_OK;
+  });
+}
+
+pard_status pard_set_draft_logits(pard_ctx* c, const float* z, int32_t sample, float temperature, uint64_t seed,
+                                  uint64_t step, int32_t* d_out, void* stream) {
+  if (!c || !z || !d_out) return fail(PARD_ERR_ARG, "null argument");
+  if (!c->prefilled) return fail(PARD_ERR_STATE, "pard_set_draft_logits before pard_prefill");
+  if (c->K == 0) return fail(PARD_ERR_STATE, "pard_set_draft_logits with K = 0 (no draft)");
+  if (sample && !(temperature > 0.f)) return fail(PARD_ERR_ARG, "temperature must be > 0 when sampling");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  c->launches = 0;
+  return guarded([&]() -> pard_status {
+    const int B = c->batch, K = c->K, V = c->D.vocab;
+    set_call(c, seed, step, temperature > 0.f ? temperature : 1.0f, sample, s);
+    CK(cudaMemcpyAsync(c->dlogits, z, (size_t)B * K * V * 4, cudaMemcpyDeviceToDevice, s));
+    launch_row_stats(c->dlogits, B * K, V, c->D.w_tiles, c->D.MC, c->call, STREAM_DRAFT, K, c->stats_d, c->stats_id,
+                     s);
+    SelectArgs sa;
+    std::memset(&sa, 0, sizeof(sa));
+    sa.mode = SEL_DRAFT_GIVEN;
+    sa.batch = B; sa.K = K; sa.w_tiles = c->D.w_tiles; sa.m_cap = c->D.MC; sa.vocab = V;
+    sa.stats = c->stats_d; sa.stats_i = c->stats_id; sa.call = c->call; sa.st = c->st; sa.out = d_out;
+    launch_select(sa, s, false);
+    c->launches += 2;
+    c->last_draft_sampled = sample != 0;
     return PARD_OK;
   });
 }
@@ -1230,16 +1117,23 @@ pard_status pard_set_mask_ids(pard_ctx* c, const int32_t* h_ids, int32_t n, void
   });
 }
 
-pard_status pard_set_fused_pass(pard_ctx* c, int32_t enable) {
-  if (!c) return fail(PARD_ERR_ARG, "null context");
-  c->fwd_enabled = enable != 0;
-  if (!c->fwd_enabled)
-    for (auto& row : c->fwd)
-      for (auto& t : row) t.ok = false;
-  return PARD_OK;
+pard_status pard_attention_paths(pard_ctx* c, uint32_t* h_bits, void* stream) {
+  if (!c || !h_bits) return fail(PARD_ERR_ARG, "null argument");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return guarded([&]() -> pard_status {
+    CK(cudaStreamSynchronize(s));
+    CK(cudaMemcpy(h_bits, c->paths, 4, cudaMemcpyDeviceToHost));
+    CK(cudaMemset(c->paths, 0, 4));
+    return PARD_OK;
+  });
 }
 
-int32_t pard_fused_pass_used(pard_ctx* c) { return c && c->fwd_used ? 1 : 0; }
+pard_status pard_set_attention_split_cap(pard_ctx* c, int32_t cap) {
+  if (!c) return fail(PARD_ERR_ARG, "null context");
+  if (cap < 0 || cap > kMaxAttnSplit) return fail(PARD_ERR_ARG, "attention split cap outside [0, 16]");
+  c->attn_split_cap = cap == 0 ? kMaxAttnSplit : cap;
+  return PARD_OK;
+}
 
 void pard_destroy(pard_ctx* c) { delete c; }
 

@@ -8,7 +8,7 @@
 // Work unit: one sequence, one KV head, a block of rows times the query
 // heads that share the KV head (<= 64 query vectors, 16 per warp), and one
 // share of the key range.  The key range is split over the CTAs of one
-// thread-block cluster (<= 8); each CTA walks its 32-key chunks with K/V
+// thread-block cluster (<= 16); each CTA walks its 32-key chunks with K/V
 // pages double-buffered in shared memory (cp.async), computes S = Q K^T and
 // O += P V on the tensor cores (mma.sync m16n8k16, fp16 inputs, fp32
 // accumulators: Q and P rounded to fp16, the bf16 K/V converted to fp16 in
@@ -71,6 +71,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
   const uint32_t recv_off = ((ring_used > part_bytes ? ring_used : part_bytes) + 127) & ~127u;
   const uint32_t recv_bytes = NS * (uint32_t)cnt * LD * 4;
   const bool push = NS > 1 && recv_off + recv_bytes <= (uint32_t)C::kKV;
+  if (a.paths && rank == 0 && threadIdx.x == 0)
+    atomicOr(a.paths, (NS == 1 ? 0u : push ? kAttnPathPush : kAttnPathPull) | (1u << (kAttnPathSplit0 + NS)));
   // every thread's partial writes, ordered before the async-proxy reads of
   // the bulk copies below, and every warp's partial in shared memory
   fence_proxy_async_smem();

@@ -1,7 +1,6 @@
 // Shared device code of the paged multi-query-position GQA attention: the
 // per-(sequence, kv head, row block) partial over a range of 32-key chunks on
-// the tensor cores.  Included by the cluster attention kernel (attention.cu)
-// and the persistent decode kernel (fwd_kernel.cuh).
+// the tensor cores.  Included by the cluster attention kernel (attention.cu).
 #pragma once
 
 #include <cuda_fp16.h>
@@ -14,7 +13,7 @@ namespace pard {
 constexpr int kAttnThreads = 128;  // 4 warps x 16 query vectors
 constexpr int kMaxQV = kMaxQVRows;
 constexpr int kKeyChunk = 32;
-constexpr int kMaxCluster = 16;  // key splits of one work unit (clusters above 8 are non-portable)
+constexpr int kMaxCluster = kMaxAttnSplit;  // key splits of one work unit (clusters above 8 are non-portable)
 constexpr int kAttnPageCache = 512;  // page ids of one work unit's key range held in shared memory
 
 // Shared memory of one work unit: NBUF K/V chunk buffers (a ring, NBUF - 1
@@ -273,7 +272,7 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
   wait_q();
 
   // ---- second wave of loads: Q ----
-  // q is rewritten by every layer, by other CTAs of a persistent grid: L2 loads
+  // q is rewritten by every layer (by the previous kernel): L2 loads
   constexpr int kQIter = kMaxQV * (HD / 4) / kAttnThreads;  // 8 or 16 float4 per thread
   constexpr int kQGroup = kQIter < 8 ? kQIter : 8;
 #pragma unroll 1

@@ -308,6 +308,12 @@ __device__ __forceinline__ float uniform_open01(uint32_t x) {
   return ((float)(x >> 9) + 0.5f) * 1.1920928955078125e-07f;
 }
 __device__ __forceinline__ float gumbel(uint32_t x) { return -logf(-logf(uniform_open01(x))); }
+// Gumbel-max score of vocabulary entry v with logit x at temperature T: the
+// categorical draw from softmax(x / T) is the entry with the largest score.
+__device__ __forceinline__ float gumbel_score(float x, float T, uint64_t seed, uint32_t stream, uint64_t step,
+                                              uint32_t b, uint32_t i, uint32_t v) {
+  return x / T + gumbel(philox_word(seed, stream, step, b, i, v));
+}
 
 enum : uint32_t { STREAM_DRAFT = 0, STREAM_ACCEPT = 1, STREAM_BONUS = 2 };
 

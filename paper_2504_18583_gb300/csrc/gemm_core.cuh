@@ -1,6 +1,5 @@
-// Shared device code of the weight-streaming GEMM: tile configuration, the
-// fused epilogues and the split-K finish.  Included by the per-phase GEMM
-// kernel (gemm.cu) and the persistent decode kernel (fwd.cu).
+// Device code of the weight-streaming GEMM (gemm.cu): tile configuration,
+// the fused epilogues and the split-K finish.
 #pragma once
 
 #include <climits>
@@ -124,7 +123,7 @@ static __device__ __forceinline__ EpiPre epi_pre(const GemmArgs& a, int w_tile, 
   if (a.mode == MODE_RESID) {
     const int n0 = w_tile * kTileN + c16;
     if (mr < M && n0 + 16 <= a.seg_rows[0] && (reinterpret_cast<uintptr_t>(a.g_next) & 15) == 0) {
-      // L2: other CTAs of a persistent grid update h
+      // L2 loads: h was written by the previous kernel's CTAs
       const float4* hp = reinterpret_cast<const float4*>(a.h + (size_t)mr * a.h_ld + n0);
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
@@ -359,9 +358,8 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
         if (m < M && valid) {
           const int ri = S.ri[kEpiTok + j];
           if (ri >= 0) {
-            const uint32_t w = philox_word(a.call->seed, (uint32_t)a.gumbel_stream, a.call->step,
-                                           (uint32_t)S.ri[2 * kEpiTok + j], (uint32_t)ri, (uint32_t)vi);
-            gv = x[j] / T + gumbel(w);
+            gv = gumbel_score(x[j], T, a.call->seed, (uint32_t)a.gumbel_stream, a.call->step,
+                              (uint32_t)S.ri[2 * kEpiTok + j], (uint32_t)ri, (uint32_t)vi);
             gi = vi;
           }
         }
@@ -408,103 +406,6 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
 }
 
 
-// Finish one segment [ub, ue) of tile t whose fp32 accumulator (hi/lo token
-// columns) sits at TMEM address tbase: the whole tile goes straight to the
-// epilogue; a partial tile writes its partial and the last CTA to arrive sums
-// all partials in CTA order and runs the epilogue.  Collective over the 128
-// epilogue threads.
-template <int TT>
-__device__ void epi_segment(const GemmArgs& a, long t, long ub, long ue, long u0, long U, long G, long c,
-                            uint32_t tbase, int w_tile, int tok_base, int fr, int et, int M, const EpiSmem& S,
-                            int* bcast) {
-  using C = GemmCfg<TT>;
-  const bool whole = (ub == t * a.kc) && (ue == (t + 1) * a.kc);
-  if (whole) {
-#pragma unroll 1
-    for (int ch = 0; ch < C::kChunks; ++ch) {
-      uint32_t r[32];
-      tmem_ld32(tbase + ch * 32, r);
-      float v[kEpiTok];
-#pragma unroll
-      for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
-      epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S,
-                epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M));
-    }
-  } else {
-    const int slot = (ub == u0) ? 0 : 1;
-    float* mine = a.partials + ((size_t)c * 2 + slot) * (kTileN * TT);
-#pragma unroll 1
-    for (int ch = 0; ch < C::kChunks; ++ch) {
-      uint32_t r[32];
-      tmem_ld32(tbase + ch * 32, r);
-      float4* dst = reinterpret_cast<float4*>(mine + ((size_t)ch * kTileN + fr) * kEpiTok);
-#pragma unroll
-      for (int j4 = 0; j4 < 4; ++j4)
-        dst[j4] = make_float4(__uint_as_float(r[8 * j4 + 0]) + __uint_as_float(r[8 * j4 + 1]),
-                              __uint_as_float(r[8 * j4 + 2]) + __uint_as_float(r[8 * j4 + 3]),
-                              __uint_as_float(r[8 * j4 + 4]) + __uint_as_float(r[8 * j4 + 5]),
-                              __uint_as_float(r[8 * j4 + 6]) + __uint_as_float(r[8 * j4 + 7]));
-    }
-    // the result-independent loads of the finishing epilogue go out now, so
-    // the CTA that turns out to finish the tile does not wait for them
-    const EpiPre pre0 = epi_pre(a, w_tile, tok_base, et, M);
-    // the barrier orders every thread's partial before the one acq_rel
-    // arrival (cumulative), which also acquires the earlier arrivals' partials
-    epi_bar();
-    const long cf = owner_of(t * a.kc, U, G), cl = owner_of((t + 1) * a.kc - 1, U, G);
-    if (et == 0) {
-      const int old = atom_add_acq_rel(&a.counters[t], 1);
-      bcast[0] = (old == (int)(cl - cf)) ? 1 : 0;
-    }
-    epi_bar();
-    if (bcast[0]) {
-#pragma unroll 1
-      for (int ch = 0; ch < C::kChunks; ++ch) {
-        uint32_t r[32];
-        tmem_ld32(tbase + ch * 32, r);
-        float v[kEpiTok];
-#pragma unroll
-        for (int j = 0; j < kEpiTok; ++j) v[j] = 0.f;
-        // contributors in CTA order, two partial tiles requested per round trip
-        for (long cc0 = cf; cc0 <= cl; cc0 += 2) {
-          float4 pv[2][4];
-#pragma unroll
-          for (int q4 = 0; q4 < 2; ++q4) {
-            const long cc = cc0 + q4;
-            if (cc <= cl && cc != c) {
-              const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
-              const float4* p = reinterpret_cast<const float4*>(
-                  a.partials + ((size_t)cc * 2 + sl) * (kTileN * TT) + ((size_t)ch * kTileN + fr) * kEpiTok);
-#pragma unroll
-              for (int j4 = 0; j4 < 4; ++j4) pv[q4][j4] = __ldcg(p + j4);
-            }
-          }
-#pragma unroll
-          for (int q4 = 0; q4 < 2; ++q4) {
-            const long cc = cc0 + q4;
-            if (cc > cl) break;
-            if (cc == c) {
-#pragma unroll
-              for (int j = 0; j < kEpiTok; ++j) v[j] += __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
-            } else {
-#pragma unroll
-              for (int j4 = 0; j4 < 4; ++j4) {
-                v[4 * j4 + 0] += pv[q4][j4].x;
-                v[4 * j4 + 1] += pv[q4][j4].y;
-                v[4 * j4 + 2] += pv[q4][j4].z;
-                v[4 * j4 + 3] += pv[q4][j4].w;
-              }
-            }
-          }
-        }
-        epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S,
-                  ch == 0 ? pre0 : epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M));
-      }
-      if (et == 0) a.counters[t] = 0;
-    }
-  }
-}
-
 // Bounded wait until *p >= target, with acquire semantics on success.
 __device__ __forceinline__ bool wait_count(const int* p, int target, volatile int* abort) {
   if (ld_acquire_s32(p) >= target) return true;
@@ -524,8 +425,7 @@ __device__ __forceinline__ bool wait_count(const int* p, int target, volatile in
 // one release increment of the tile's counter and move on without a round
 // trip.  cf waits for the cl - cf increments, pulls every partial into the
 // ring with one bulk copy each (a single round trip for the whole tile) and
-// sums in CTA order, itself first: the same order, so the same sums, as the
-// last-arriver scheme of epi_segment.  pre0: epi_pre of the segment's first
+// sums in CTA order, itself first (deterministic).  pre0: epi_pre of the segment's first
 // chunk, taken by the caller before the accumulator was ready; only read for
 // a whole tile or by cf.  ring/ring_bytes: the stage ring; fx: an mbarrier
 // used once per launch; fx_armed: set while its copies are in flight.

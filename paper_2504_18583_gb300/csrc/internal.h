@@ -101,7 +101,14 @@ struct AttnArgs {
   __nv_bfloat16* x_out;       // packed [2*rows][hq*hd] hi/lo
   int x_rows;
   uint32_t* status;
+  uint32_t* paths;            // combine paths taken (kAttnPath* bits, OR-ed; null: not recorded)
 };
+
+// Attention combine paths recorded in AttnArgs::paths: push or pull combine
+// of the key splits, and bit kAttnPathSplit0 + n for clusters of n CTAs.
+constexpr uint32_t kAttnPathPush = 1u << 0;
+constexpr uint32_t kAttnPathPull = 1u << 1;
+constexpr int kAttnPathSplit0 = 3;
 
 // Per-sequence decode state, in the workspace.
 struct DevState {
@@ -153,7 +160,7 @@ struct EmbedArgs {
 enum { EMB_PREFILL = 0, EMB_DRAFT = 1, EMB_VERIFY = 2, EMB_DRAFT_SEQ = 3 };
 
 struct SelectArgs {
-  int mode;          // SEL_DRAFT, SEL_FIRST, SEL_NORM_ONLY, SEL_DRAFT_SEQ
+  int mode;          // SEL_DRAFT, SEL_FIRST, SEL_NORM_ONLY, SEL_DRAFT_SEQ, SEL_DRAFT_GIVEN
   int batch, K, w_tiles, m_cap, vocab;
   int seq_i;         // SEL_DRAFT_SEQ: the candidate this pass picks
   const float4* stats;
@@ -165,7 +172,8 @@ struct SelectArgs {
   const int* plen;   // first token: prompt lengths
   int n_new;
 };
-enum { SEL_DRAFT = 0, SEL_FIRST = 1, SEL_NORM_ONLY = 2, SEL_DRAFT_SEQ = 3 };
+// SEL_DRAFT_GIVEN: candidates from given draft logits rows b * K + i
+enum { SEL_DRAFT = 0, SEL_FIRST = 1, SEL_NORM_ONLY = 2, SEL_DRAFT_SEQ = 3, SEL_DRAFT_GIVEN = 4 };
 
 struct AcceptArgs {
   int batch, K, w_tiles, m_cap, vocab;
@@ -181,39 +189,13 @@ struct AcceptArgs {
   int* emitted;
   int* kv_slots;
   int* n_emit;
+  uint32_t* status;        // sticky device status word (null: none)
 };
 
-// Persistent decode pass: one launch runs every phase of every layer.
-enum PhaseType : int { PH_GEMM = 0, PH_ATTN = 1 };
-struct Phase {
-  int type;
-  int dep;            // phase whose completion this phase's inputs need (-1: none)
-  int attn_groups;    // PH_ATTN: (sequence, kv head, row block) groups
-  int attn_split;     // PH_ATTN: key splits per group
-  GemmArgs g;         // PH_GEMM (packed weights, one token tile)
-  AttnArgs at;        // PH_ATTN
-};
-struct FwdArgs {
-  const Phase* phases;   // device array
-  int n_phases;
-  unsigned* done;        // per-phase completion counters, monotonic over launches
-  unsigned target;       // a phase is complete when done[p] reaches target (launch count x grid)
-  float* attn_part;      // [groups * split][64][hd + 2] attention partials
-  int* attn_cnt;         // [groups] arrival counters (left at zero)
-  uint32_t* status;
-  const int* m_dev;
-  int m_cap;
-};
-constexpr int kFwdMaxAttnItems = 1024;  // (group, split) attention items of one persistent pass
 constexpr int kMaxQVRows = 64;          // query vectors of one attention work unit
-constexpr int kFwdTT = 16;              // persistent pass: token tile (rows of one pass, at most)
-constexpr int kFwdMaxSplit = 8;         // persistent pass: key splits per attention group
-constexpr int kFwdPrefetch = 8;         // persistent pass: weight units each CTA keeps requested into L2 ahead
-constexpr int kFwdPrefetchMax = 8;      // ... and at most this many while its ring waits on a phase
+constexpr int kMaxAttnSplit = 16;       // key splits (CTAs of one cluster) of one attention work unit
 
-// launchers (gemm.cu, attention.cu, misc.cu, fwd.cu)
-int fwd_smem_bytes(int hd);
-cudaError_t launch_fwd(const FwdArgs& f, int hd, int group, int grid, cudaStream_t s);
+// launchers (gemm.cu, attention.cu, misc.cu)
 void launch_embed(const EmbedArgs& a, int grid, cudaStream_t s, bool pdl);
 void launch_gather_rows(const __nv_bfloat16* x, int x_rows, const float* ssq, int ssq_tiles, int m_cap_src, int src_row,
                         __nv_bfloat16* xg, int xg_rows, float* ssqg, int m_cap_dst, int dst_row, int d, cudaStream_t s,
@@ -223,7 +205,7 @@ void launch_select(const SelectArgs& a, cudaStream_t s, bool pdl);
 void launch_accept_greedy(const AcceptArgs& a, cudaStream_t s, bool pdl);
 void launch_accept_sample(const AcceptArgs& a, cudaStream_t s, bool pdl);
 void launch_row_stats(const float* logits, int rows, int vocab, int w_tiles, int m_cap, const CallArgs* call,
-                      float4* stats, int2* stats_i, cudaStream_t s);
+                      int gumbel_stream, int rows_per_seq, float4* stats, int2* stats_i, cudaStream_t s);
 void launch_set_call(CallArgs* dst, CallArgs v, cudaStream_t s, bool pdl);
 void launch_copy_i32(const int* src, int* dst, int n, cudaStream_t s, bool pdl);
 void launch_copy_f32(const float* src, float* dst, size_t n, cudaStream_t s, bool pdl);

@@ -290,7 +290,7 @@ __global__ void __launch_bounds__(256) select_kernel(const __grid_constant__ Sel
     return;
   }
   a.st.dnorm[b * a.st.kmax + i] = make_float2(r.mx, r.se);
-  if (a.mode == SEL_DRAFT || a.mode == SEL_DRAFT_SEQ) {
+  if (a.mode == SEL_DRAFT || a.mode == SEL_DRAFT_SEQ || a.mode == SEL_DRAFT_GIVEN) {
     a.st.d[b * a.st.kmax + i] = tok;
     if (a.out) a.out[b * a.K + i] = tok;
   }
@@ -352,6 +352,11 @@ __global__ void __launch_bounds__(256) accept_greedy_kernel(const __grid_constan
   if (threadIdx.x != 0) return;
   int acc = 0;
   while (acc < a.K && a.st.d[b * a.st.kmax + acc] == s_arg[acc]) ++acc;
+  // a candidate outside the vocabulary never equals an argmax (rejected); flag it
+  for (int i = 0; i < a.K && a.status; ++i) {
+    const int di = a.st.d[b * a.st.kmax + i];
+    if (di < 0 || di >= a.vocab) set_status(a.status, ST_BAD_TOKEN);
+  }
   int em[17];
   for (int j = 0; j < acc; ++j) em[j] = a.st.d[b * a.st.kmax + j];
   em[acc] = s_arg[acc];
@@ -379,6 +384,12 @@ __global__ void __launch_bounds__(256) accept_test_kernel(const __grid_constant_
   int j = a.K;
   for (int i = 0; i < a.K; ++i) {
     const int di = a.st.d[b * a.st.kmax + i];
+    if (di < 0 || di >= a.vocab) {
+      // a candidate outside the vocabulary has no probability: rejected
+      if (a.status) set_status(a.status, ST_BAD_TOKEN);
+      j = i;
+      break;
+    }
     const float yv = a.logits[((size_t)b * (a.K + 1) + i) * a.vocab + di];
     const float p = expf(yv / T - s_norm[i].x / T) / s_norm[i].y;
     const float2 zn = a.st.dnorm[b * a.st.kmax + i];
@@ -494,30 +505,49 @@ void launch_accept_sample(const AcceptArgs& a, cudaStream_t s, bool pdl) {
   PARD_LAUNCH(resample_kernel, a.batch * kResampleSplit, 256, 0, s, true, a);
 }
 
-// Tile statistics of given logits rows (same layout as the LM-head epilogue).
+// Tile statistics of given logits rows (same layout as the LM-head
+// epilogue): per 128-entry tile the max and argmax, the sum of exp((x - max)/T)
+// and, when gumbel_stream >= 0 and the call samples, the Gumbel-max winner of
+// the tile for row m = b * rows_per_seq + i (Philox row i of sequence b), the
+// draw the LM-head epilogue makes for a draft row.
 __global__ void __launch_bounds__(128) row_stats_kernel(const float* logits, int vocab, int m_cap, const CallArgs* call,
-                                                        float4* stats, int2* stats_i) {
+                                                        int gumbel_stream, int rows_per_seq, float4* stats,
+                                                        int2* stats_i) {
   pdl_wait();
   const int t = blockIdx.x, m = blockIdx.y;
   const int v = t * 128 + threadIdx.x;
   const float T = call->temp;
   const bool valid = v < vocab;
+  const bool gumb = gumbel_stream >= 0 && call->sample != 0;
   const float x = valid ? logits[(size_t)m * vocab + v] : -INFINITY;
-  __shared__ float s_v[4];
-  __shared__ int s_i[4];
+  __shared__ float s_v[4], s_g[4];
+  __shared__ int s_i[4], s_gi[4];
   __shared__ float s_m;
   float mv = x;
   int mi = valid ? v : INT_MAX;
   warp_argmax(mv, mi);
+  float gv = -INFINITY;
+  int gi = INT_MAX;
+  if (gumb && valid) {
+    gv = gumbel_score(x, T, call->seed, (uint32_t)gumbel_stream, call->step, (uint32_t)(m / rows_per_seq),
+                      (uint32_t)(m % rows_per_seq), (uint32_t)v);
+    gi = v;
+  }
+  if (gumb) warp_argmax(gv, gi);
   const int w = threadIdx.x >> 5;
-  if ((threadIdx.x & 31) == 0) { s_v[w] = mv; s_i[w] = mi; }
+  if ((threadIdx.x & 31) == 0) { s_v[w] = mv; s_i[w] = mi; s_g[w] = gv; s_gi[w] = gi; }
   __syncthreads();
   if (threadIdx.x == 0) {
     float bv = s_v[0];
     int bi = s_i[0];
     for (int k = 1; k < 4; ++k) argmax_merge(bv, bi, s_v[k], s_i[k]);
+    float bg = s_g[0];
+    int bgi = s_gi[0];
+    for (int k = 1; k < 4; ++k) argmax_merge(bg, bgi, s_g[k], s_gi[k]);
     s_m = bv;
     s_i[0] = bi;
+    s_g[0] = bg;
+    s_gi[0] = bgi;
   }
   __syncthreads();
   const float mxv = s_m;
@@ -528,14 +558,16 @@ __global__ void __launch_bounds__(128) row_stats_kernel(const float* logits, int
   if ((threadIdx.x & 31) == 0) s_v[w] = e;
   __syncthreads();
   if (threadIdx.x == 0) {
-    stats[(size_t)t * m_cap + m] = make_float4(mxv, ((s_v[0] + s_v[1]) + s_v[2]) + s_v[3], -INFINITY, 0.f);
-    stats_i[(size_t)t * m_cap + m] = make_int2(arg, -1);
+    stats[(size_t)t * m_cap + m] =
+        make_float4(mxv, ((s_v[0] + s_v[1]) + s_v[2]) + s_v[3], gumb ? s_g[0] : -INFINITY, 0.f);
+    stats_i[(size_t)t * m_cap + m] = make_int2(arg, gumb ? s_gi[0] : -1);
   }
 }
 
 void launch_row_stats(const float* logits, int rows, int vocab, int w_tiles, int m_cap, const CallArgs* call,
-                      float4* stats, int2* stats_i, cudaStream_t s) {
-  PARD_LAUNCH(row_stats_kernel, dim3(w_tiles, rows), 128, 0, s, false, logits, vocab, m_cap, call, stats, stats_i);
+                      int gumbel_stream, int rows_per_seq, float4* stats, int2* stats_i, cudaStream_t s) {
+  PARD_LAUNCH(row_stats_kernel, dim3(w_tiles, rows), 128, 0, s, false, logits, vocab, m_cap, call, gumbel_stream,
+              rows_per_seq > 0 ? rows_per_seq : 1, stats, stats_i);
 }
 
 __global__ void set_call_kernel(CallArgs* dst, CallArgs v) {

@@ -152,7 +152,7 @@ extern "C" pard_status pard_accept_noalloc(const float* d_target_logits, const f
     e = cudaMemcpyAsync(st.d, d_draft, (size_t)batch * K * 4, cudaMemcpyDeviceToDevice, s);
     if (e != cudaSuccess) throw e;
     launch_set_call(call, CallArgs{seed, step, temperature, sample ? 1 : 0, K, 0}, s, false);
-    launch_row_stats(d_target_logits, batch * (K + 1), vocab, tiles, kNaRowsT, call, stats_t, stats_it, s);
+    launch_row_stats(d_target_logits, batch * (K + 1), vocab, tiles, kNaRowsT, call, -1, 1, stats_t, stats_it, s);
     AcceptArgs a;
     memset(&a, 0, sizeof(a));
     a.batch = batch; a.K = K; a.w_tiles = tiles; a.m_cap = kNaRowsT; a.vocab = vocab;
@@ -161,7 +161,7 @@ extern "C" pard_status pard_accept_noalloc(const float* d_target_logits, const f
     a.page_table = nullptr; a.pt_ld = 0; a.page_size = 16;
     a.accept_len = d_accept_len; a.emitted = d_emitted; a.kv_slots = nullptr; a.n_emit = nullptr;
     if (sample) {
-      launch_row_stats(d_draft_logits, batch * K, vocab, tiles, kNaRowsD, call, stats_d, stats_id, s);
+      launch_row_stats(d_draft_logits, batch * K, vocab, tiles, kNaRowsD, call, -1, 1, stats_d, stats_id, s);
       SelectArgs sa;
       memset(&sa, 0, sizeof(sa));
       sa.mode = SEL_NORM_ONLY;

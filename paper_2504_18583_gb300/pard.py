@@ -67,11 +67,16 @@ def lib() -> ctypes.CDLL:
         L.pard_verify.argtypes = [vp, vp, f32, vp, vp]
         L.pard_accept_commit.argtypes = [vp, i32, f32, u64, u64, vp, vp, vp, vp, vp]
         L.pard_set_logits.argtypes = [vp, vp, vp, vp, f32, vp]
+        L.pard_set_draft_logits.argtypes = [vp, vp, i32, f32, u64, u64, vp, vp]
         L.pard_get_state.argtypes = [vp, vp, vp, vp, vp]
         L.pard_read_kv.argtypes = [vp, i32, i32, i32, vp, i32, vp, vp, vp]
         L.pard_last_status.argtypes = [vp, P(ctypes.c_uint32), vp]
         L.pard_accept_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, f32, u64, u64, vp, vp, vp]
         L.pard_accept_noalloc.restype = ctypes.c_int
+        L.pard_attention_paths.argtypes = [vp, P(ctypes.c_uint32), vp]
+        L.pard_attention_paths.restype = ctypes.c_int
+        L.pard_set_attention_split_cap.argtypes = [vp, i32]
+        L.pard_set_attention_split_cap.restype = ctypes.c_int
         L.pard_unpack_weights.argtypes = [vp, vp]
         L.pard_unpack_weights.restype = ctypes.c_int
         L.pard_launch_count.argtypes = [vp]
@@ -80,13 +85,9 @@ def lib() -> ctypes.CDLL:
         L.pard_last_error.restype = ctypes.c_char_p
         L.pard_destroy.argtypes = [vp]
         L.pard_destroy.restype = None
-        L.pard_set_fused_pass.argtypes = [vp, i32]
-        L.pard_set_fused_pass.restype = ctypes.c_int
-        L.pard_fused_pass_used.argtypes = [vp]
-        L.pard_fused_pass_used.restype = i32
         for name in ("pard_load_weights", "pard_prefill", "pard_draft", "pard_draft_sequential", "pard_verify",
                      "pard_accept_commit", "pard_set_mask_ids", "pard_selftest_stalled_wait", "pard_cod_select",
-                     "pard_set_logits", "pard_get_state", "pard_read_kv", "pard_last_status"):
+                     "pard_set_logits", "pard_set_draft_logits", "pard_get_state", "pard_read_kv", "pard_last_status"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -266,6 +267,11 @@ class PardEngine:
         _check(lib().pard_set_logits(self.ctx, target_logits.data_ptr(), _ptr(draft_logits), draft.data_ptr(),
                                      temperature, self.stream.cuda_stream), "pard_set_logits")
 
+    def set_draft_logits(self, draft_logits, out, sample=False, temperature=1.0, seed=0, step=0):
+        """Candidates from given draft logits [B, K, V] into out['draft'] (pard_set_draft_logits)."""
+        _check(lib().pard_set_draft_logits(self.ctx, draft_logits.data_ptr(), int(sample), temperature, seed, step,
+                                           out["draft"].data_ptr(), self.stream.cuda_stream), "pard_set_draft_logits")
+
     def state(self):
         B = max(self.batch, 1)
         n, g, d = (ctypes.c_int32 * B)(), (ctypes.c_int32 * B)(), (ctypes.c_int32 * B)()
@@ -301,10 +307,14 @@ class PardEngine:
     def launch_count(self) -> int:
         return lib().pard_launch_count(self.ctx)
 
-    def set_fused_pass(self, enable: bool) -> None:
-        """Persistent single-kernel forward for small passes (default off); applies from the next prefill."""
-        _check(lib().pard_set_fused_pass(self.ctx, 1 if enable else 0), "pard_set_fused_pass")
+    def attention_paths(self) -> int:
+        """Attention combine forms run since the last call (bit 0 push, bit 1
+        pull, bit 3 + n: clusters of n CTAs); the record is cleared."""
+        bits = ctypes.c_uint32(0)
+        _check(lib().pard_attention_paths(self.ctx, ctypes.byref(bits), self.stream.cuda_stream),
+               "pard_attention_paths")
+        return bits.value
 
-    def fused_pass_used(self) -> bool:
-        """True when the last draft / verify ran as one persistent kernel."""
-        return bool(lib().pard_fused_pass_used(self.ctx))
+    def set_attention_split_cap(self, cap: int) -> None:
+        """At most `cap` key splits (CTAs of one cluster) per attention unit; 0: the default 16."""
+        _check(lib().pard_set_attention_split_cap(self.ctx, int(cap)), "pard_set_attention_split_cap")

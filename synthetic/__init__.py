@@ -121,11 +121,15 @@ class Workload:
     page_size: int
     seed: int
     norm_jitter: float = 0.0             # 0: norm gains are 1.0
+    prompt_lens_given: Optional[Tuple[int, ...]] = None  # one length per sequence (overrides the two above)
 
     def replace(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
 
     def prompt_lens(self) -> List[int]:
+        if self.prompt_lens_given is not None:
+            assert len(self.prompt_lens_given) == self.batch
+            return [int(x) for x in self.prompt_lens_given]
         if self.prompt_len is not None:
             return [self.prompt_len] * self.batch
         lo, hi = self.prompt_len_range

@@ -15,10 +15,13 @@ import numpy as np
 import oracle
 import synthetic as S
 from oracle import pard as OP
-from oracle.philox import STREAM_ACCEPT, raw_words, uniform01
+from oracle.philox import STREAM_ACCEPT, STREAM_BONUS, STREAM_DRAFT, raw_words, uniform01
 
 LOGIT_TOL = 3e-2
 MARGIN = 5e-2
+# Gumbel noise is -log(-log u) on both sides, with different log routines:
+# allow a few fp32 ulps of the largest noise values (|G| < 20)
+GUMBEL_EPS = 1e-5
 
 
 def margin(row: np.ndarray) -> float:
@@ -26,10 +29,64 @@ def margin(row: np.ndarray) -> float:
     return float(top2[1] - top2[0])
 
 
+def gumbel_scores(logits_row: np.ndarray, T: float, seed: int, stream: int, step: int, b: int, i: int) -> np.ndarray:
+    """The oracle's Gumbel-max scores z / T + G (the categorical draw is their argmax)."""
+    z = (np.asarray(logits_row, dtype=np.float32) / np.float32(T)).astype(np.float32)
+    return (z + OP.gumbel_noise(seed, stream, step, b, i, z.shape[0])).astype(np.float32)
+
+
+def check_sampled(gpu_tok: int, scores: np.ndarray, bound: float, stats: dict, what: str) -> None:
+    """A Gumbel-max draw: each score of the GPU differs from the oracle's by at
+    most bound / 2, so where the oracle's winner leads the runner-up by more
+    than bound the GPU must draw the same token; elsewhere its token must
+    score within bound of the oracle's winner."""
+    o_tok = int(np.argmax(scores))
+    stats["sampled_checked"] = stats.get("sampled_checked", 0) + 1
+    if margin(scores) > bound:
+        assert gpu_tok == o_tok, f"{what}: gpu {gpu_tok} oracle {o_tok} margin {margin(scores):.3g} > {bound:.3g}"
+        stats["sampled_exact"] = stats.get("sampled_exact", 0) + 1
+    else:
+        assert scores[gpu_tok] >= scores[o_tok] - bound, what
+        if gpu_tok != o_tok:
+            stats["excused_tokens"] += 1
+
+
+def check_residual_draw(gpu_tok: int, y: np.ndarray, z: np.ndarray, T: float, err_y: float, err_z: float,
+                        seed: int, step: int, b: int, stats: dict, what: str) -> None:
+    """The bonus token after a rejection: a Gumbel-max draw over
+    log max(0, p - q) with Philox stream 2.  With the GPU's logits within
+    err_y / err_z of the oracle's, log p_v and log q_v move by at most
+    2 err / T, which bounds every GPU weight w_v = max(0, p_v - q_v) to
+    [w_v - s_v, w_v + s_v]; the GPU must draw the oracle's winner whenever the
+    winner's lowest possible score beats every other entry's highest."""
+    p = OP.softmax_t(y, T).astype(np.float64)
+    q = OP.softmax_t(z, T).astype(np.float64)
+    w = np.maximum(p - q, 0.0)
+    if not (w > 0).any():
+        return
+    slack = p * np.expm1(2 * err_y / T) + q * np.expm1(2 * err_z / T) + 1e-12
+    g = OP.gumbel_noise(seed, STREAM_BONUS, step, b, 0, y.shape[0]).astype(np.float64)
+    with np.errstate(divide="ignore"):
+        score = np.where(w > 0, np.log(w) + g, -np.inf)
+        hi = np.log(w + slack) + g
+        lo = np.where(w - slack > 0, np.log(np.maximum(w - slack, 1e-300)) + g, -np.inf)
+    o_tok = int(np.argmax(score))
+    others = hi.copy()
+    others[o_tok] = -np.inf
+    stats["sampled_checked"] = stats.get("sampled_checked", 0) + 1
+    if lo[o_tok] > others.max() + GUMBEL_EPS:
+        assert gpu_tok == o_tok, f"{what}: gpu {gpu_tok} oracle {o_tok}"
+        stats["sampled_exact"] = stats.get("sampled_exact", 0) + 1
+    else:
+        assert hi[gpu_tok] + GUMBEL_EPS >= lo[o_tok], what
+        if gpu_tok != o_tok:
+            stats["excused_tokens"] += 1
+
+
 class Pair:
     """GPU engine and oracle decoder on identical weights and page orders."""
 
-    def __init__(self, wl, draft_is_target: bool = False, prefill_chunk: int = 64, fused: bool = True):
+    def __init__(self, wl, draft_is_target: bool = False, prefill_chunk: int = 64):
         import torch
         from paper_2504_18583_gb300 import pard
         self.wl = wl
@@ -49,7 +106,6 @@ class Pair:
         self.eng = pard.PardEngine(wl.target, self.tw_dev, dshape, self.dw_dev, max_batch=wl.batch, max_k=wl.K,
                                    max_ctx=max_ctx, n_pages=n_pages, prefill_chunk=prefill_chunk,
                                    page_order_target=self.order_t, page_order_draft=self.order_d)
-        self.eng.set_fused_pass(fused)
         self.torch = torch
         self.stats = dict(excused_tokens=0, checked_tokens=0, max_logit_err=0.0, max_draft_logit_err=0.0)
 
@@ -60,6 +116,13 @@ class Pair:
         for b in range(self.wl.batch):
             if not self.wl.sample:
                 check_token(int(first_g[b]), self.oracle.prefill_logits[b], self.stats, f"first token seq {b}")
+            else:
+                # drawn from the target's last prompt row (stream 2, step 0); the
+                # GPU's prefill logits are within LOGIT_TOL of the oracle's
+                T = self.wl.temperature
+                sc = gumbel_scores(self.oracle.prefill_logits[b], T, seed, STREAM_BONUS, 0, b, 0)
+                check_sampled(int(first_g[b]), sc, 2 * LOGIT_TOL / T + GUMBEL_EPS, self.stats,
+                              f"sampled first token seq {b}")
             if int(first_g[b]) != int(first_o[b]):
                 self.stats["excused_tokens"] += 1
                 self.oracle.force_first(b, int(first_g[b]))
@@ -152,3 +215,77 @@ def greedy_step(P: Pair, step: int, inject=None, sequential: bool = False):
         assert np.array_equal(slots_gpu[b], slots_or[b]), f"kv slots step {step} seq {b}"
         assert n_emit[b] == nout[b]
     return dict(a=a_gpu, emitted=em_gpu, slots=slots_gpu, d=d_gpu, y=y_gpu, z=z_gpu)
+
+
+def sampling_step(P: Pair, step: int, seed: int) -> dict:
+    """One teacher-forced speculative-sampling step (Section 2.2 with the
+    draft of Eq. 6 at temperature T): draft logits, verify logits within
+    LOGIT_TOL; the draft's Gumbel-max candidates, the accept / reject
+    decisions and the bonus draw against the oracle's on the same Philox
+    streams wherever the margins are clear; KV slots bit-exact.  The oracle
+    is then committed with the GPU's tokens."""
+    wl, K, T = P.wl, P.wl.K, P.wl.temperature
+    out = P.eng.alloc_step_outputs(want_logits=True)
+    P.eng.draft(out, True, T, seed, step)
+    d_g = out["draft"].cpu().numpy()
+    z_g = out["draft_logits"].cpu().numpy()
+    d_o, z_o = P.oracle.draft(step, seed)
+    for b in P.active():
+        for i in range(K):
+            err = float(np.abs(z_g[b, i] - z_o[b, i]).max())
+            P.stats["max_draft_logit_err"] = max(P.stats["max_draft_logit_err"], err)
+            assert err <= LOGIT_TOL, f"draft logits step {step} seq {b} row {i}: {err}"
+            sc = gumbel_scores(z_o[b, i], T, seed, STREAM_DRAFT, step, b, i)
+            assert int(d_o[b, i]) == int(np.argmax(sc))
+            check_sampled(int(d_g[b, i]), sc, 2 * err / T + GUMBEL_EPS, P.stats,
+                          f"sampled draft step {step} seq {b} row {i}")
+    P.eng.verify(out, None, T)
+    y_g = out["logits"].cpu().numpy()
+    y_o = P.oracle.verify(d_g)
+    for b in P.active():
+        err = float(np.abs(y_g[b] - y_o[b]).max())
+        P.stats["max_logit_err"] = max(P.stats["max_logit_err"], err)
+        assert err <= LOGIT_TOL, f"verify logits step {step} seq {b}: {err}"
+    P.eng.accept_commit(out, True, T, seed, step)
+    a_g = out["accept_len"].cpu().numpy()
+    em_g = out["emitted"].cpu().numpy()
+    n_emit = out["n_emit"].cpu().numpy()
+    slots_g = out["kv_slots"].cpu().numpy()
+    acc, emitted = [], []
+    for b in range(wl.batch):
+        if P.oracle.done[b]:
+            assert a_g[b] == 0 and n_emit[b] == 0
+            acc.append(0)
+            emitted.append([])
+            continue
+        a = int(a_g[b])
+        for i in range(min(a + 1, K)):
+            p = OP.softmax_t(y_o[b, i], T)[d_g[b, i]]
+            q = OP.softmax_t(z_o[b, i], T)[d_g[b, i]]
+            u = uniform01(raw_words(seed, STREAM_ACCEPT, step, b, i, np.zeros(1, np.uint64)))[0]
+            if abs(u - p / q) > 1e-3:
+                assert (u * q < p) == (i < a), (step, b, i)
+                P.stats["decisions_checked"] = P.stats.get("decisions_checked", 0) + 1
+        take = int(n_emit[b])
+        em = [int(x) for x in em_g[b, :take]]
+        assert em[:min(a, take)] == [int(x) for x in d_g[b, :min(a, take)]]
+        a_o, _ = OP.accept_sampling(d_g[b], z_o[b], y_o[b], T, seed, step, b)
+        if a_o == a and take == a + 1:
+            err_y = float(np.abs(y_g[b, a] - y_o[b, a]).max())
+            if a == K:
+                sc = gumbel_scores(y_o[b, K], T, seed, STREAM_BONUS, step, b, 0)
+                check_sampled(em[a], sc, 2 * err_y / T + GUMBEL_EPS, P.stats, f"bonus p_K step {step} seq {b}")
+            else:
+                err_z = float(np.abs(z_g[b, a] - z_o[b, a]).max())
+                check_residual_draw(em[a], y_o[b, a], z_o[b, a], T, err_y, err_z, seed, step, b, P.stats,
+                                    f"residual draw step {step} seq {b} row {a}")
+        full = em if len(em) == a + 1 else em + [0] * (a + 1 - len(em))
+        acc.append(a)
+        emitted.append(full)
+    slots_o, nout = P.oracle.commit(acc, emitted)
+    for b in range(wl.batch):
+        if nout[b] == 0 and a_g[b] == 0 and n_emit[b] == 0:
+            continue
+        assert np.array_equal(slots_g[b], slots_o[b]), f"kv slots step {step} seq {b}"
+        assert n_emit[b] == nout[b]
+    return dict(a=a_g, emitted=em_g, d=d_g)

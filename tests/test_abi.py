@@ -68,12 +68,13 @@ def test_load_rejects_bad_shapes_before_touching_the_device():
     assert pard.lib().pard_draft_sequential(None, 0, 1.0, 0, 0, None, None, None) == -1
     assert pard.lib().pard_set_mask_ids(None, None, 0, None) == -1
     assert pard.lib().pard_selftest_stalled_wait(None, None) == -1
+    assert pard.lib().pard_set_attention_split_cap(None, 8) == -1
+    bits = ctypes.c_uint32(0)
+    assert pard.lib().pard_attention_paths(None, ctypes.byref(bits), None) == -1
     # COD: argument checks happen on the host, before any launch
     for n, K, r, r_min in ((0, 3, 0.5, 0.0), (4097, 3, 0.5, 0.0), (10, 0, 0.5, 0.0), (10, 3, 0.0, 0.0),
                            (10, 3, 1.5, 0.0), (10, 3, 0.5, -0.1)):
         assert pard.lib().pard_cod_select(n, K, r, r_min, 0, 0, None, None, None) == -1
-    assert pard.lib().pard_set_fused_pass(None, 1) == -1
-    assert pard.lib().pard_fused_pass_used(None) == 0
 
 
 def test_binding_fails_loudly_without_the_library(monkeypatch, tmp_path):

@@ -6,9 +6,9 @@ import pytest
 import oracle
 import synthetic as S
 from oracle import pard as OP
-from oracle.philox import STREAM_ACCEPT, STREAM_BONUS, raw_words, uniform01
+from oracle.philox import STREAM_ACCEPT, STREAM_BONUS, STREAM_DRAFT, raw_words, uniform01
 
-from _parity import LOGIT_TOL, MARGIN, Pair, check_token, greedy_step, margin
+from _parity import GUMBEL_EPS, LOGIT_TOL, MARGIN, Pair, check_token, greedy_step, gumbel_scores, margin, sampling_step
 
 pytestmark = pytest.mark.gpu
 
@@ -33,21 +33,19 @@ def run_greedy(P: Pair, max_steps=64, inject_fn=None, sequential=False):
     return outs
 
 
-@pytest.mark.parametrize("fused", [True, False], ids=["persistent", "per_phase"])
-def test_tiny_greedy_matches_oracle_every_step(fused):
-    """Both forward-pass paths: the persistent kernel (draft 8 rows, verify 5
-    rows; FFN 768 so every matrix takes the packed layout it needs) and one
-    kernel per phase (FFN 688: ragged row-major gate/up/down)."""
-    wl = S.WORKLOADS["tiny"]
-    if fused:
-        wl = wl.replace(target=wl.target.replace(ffn=768), draft=wl.draft.replace(ffn=768))
-    P = Pair(wl, fused=fused)
-    run_greedy(P)
-    assert P.eng.fused_pass_used() == fused
-    assert P.oracle.all_done()
-    # the generated sequence equals autoregressive greedy decoding where margins are clear
-    assert P.stats["excused_tokens"] <= P.stats["checked_tokens"] // 10
-    print("stats", P.stats)
+def test_tiny_greedy_matches_oracle_every_step():
+    """The tiny configuration (FFN 688: ragged row-major gate/up/down tiles)
+    against the oracle step by step; and with FFN 768, where every matrix
+    takes the packed layout."""
+    for ffn in (688, 768):
+        wl = S.WORKLOADS["tiny"]
+        wl = wl.replace(target=wl.target.replace(ffn=ffn), draft=wl.draft.replace(ffn=ffn))
+        P = Pair(wl)
+        run_greedy(P)
+        assert P.oracle.all_done()
+        # the generated sequence equals autoregressive greedy decoding where margins are clear
+        assert P.stats["excused_tokens"] <= P.stats["checked_tokens"] // 10
+        print("ffn", ffn, "stats", P.stats)
 
 
 def test_vanilla_sd_sequential_draft_matches_oracle_every_step():
@@ -172,8 +170,6 @@ def test_tiny_greedy_jittered_norms_batch_ragged():
     wl = wl.replace(target=wl.target.replace(ffn=768), draft=wl.draft.replace(ffn=768))
     P = Pair(wl)
     run_greedy(P)
-    # 3 x 8 draft rows exceed one persistent pass; the 3 x 5 verify rows fit
-    assert P.eng.fused_pass_used()
     print("stats", P.stats)
 
 
@@ -233,18 +229,16 @@ def test_kv_cache_holds_the_oracle_keys_and_values():
             assert np.abs(v - vo).max() <= 0.02 * max(1.0, np.abs(vo).max())
 
 
-@pytest.mark.parametrize("fused", [True, False], ids=["persistent", "per_phase"])
-def test_full_width_8b_layers_short_prompt(fused):
+def test_full_width_8b_layers_short_prompt():
     """8B-shaped target and 1B-shaped draft at full width (every GEMM,
     attention and LM-head tile count of the full models), two layers each,
     64-token prompt, three steps; K = 8 gives 16 draft rows and 9 verify rows."""
     wl = S.WORKLOADS["8b_greedy"].replace(target=S.TARGET_8B.replace(n_layers=2),
                                           draft=S.DRAFT_1B.replace(n_layers=2), prompt_len=64, n_new=20)
-    P = Pair(wl, prefill_chunk=64, fused=fused)
+    P = Pair(wl, prefill_chunk=64)
     P.prefill()
     for step in range(1, 4):
         greedy_step(P, step)
-    assert P.eng.fused_pass_used() == fused
     assert P.eng.last_status() == 0
     print("stats", P.stats)
 
@@ -344,81 +338,84 @@ def test_sampling_decisions_on_identical_logits():
 
 
 def test_sampling_end_to_end_tiny():
-    """Level 2: sampling decode end to end; GPU and oracle decisions agree
-    wherever |u - p/q| > 1e-3 and draws agree where their Gumbel margins are
-    clear; the oracle follows the GPU's tokens."""
-    wl = S.WORKLOADS["tiny"].replace(sample=True, n_new=24)
+    """Level 2: sampling decode end to end (tiny models, batch 2, ragged
+    prompts).  The sampled first token, the draft's Gumbel-max candidates,
+    the accept / reject decisions and the bonus draws agree with the
+    oracle's on the same Philox streams wherever the margins are clear (the
+    margins follow from the measured logit differences); the oracle follows
+    the GPU's tokens."""
+    wl = S.WORKLOADS["tiny"].replace(sample=True, n_new=40, batch=2, prompt_len=None, prompt_len_range=(20, 45))
     P = Pair(wl)
     seed = 11
     P.prefill(seed)
-    K = wl.K
     step = 1
-    checked = 0
-    while not P.oracle.all_done() and step < 40:
-        out = P.eng.alloc_step_outputs(want_logits=True)
-        P.eng.draft(out, True, 1.0, seed, step)
-        d_g = out["draft"].cpu().numpy()
-        z_g = out["draft_logits"].cpu().numpy()
-        d_o, z_o = P.oracle.draft(step, seed)
-        assert np.abs(z_g - z_o).max() <= LOGIT_TOL
-        P.eng.verify(out, None, 1.0)
-        y_g = out["logits"].cpu().numpy()
-        y_o = P.oracle.verify(d_g)
-        assert np.abs(y_g - y_o).max() <= LOGIT_TOL
-        P.eng.accept_commit(out, True, 1.0, seed, step)
-        a_g = int(out["accept_len"][0])
-        # decisions where clear
-        for i in range(min(a_g + 1, K)):
-            p = OP.softmax_t(y_o[0, i], 1.0)[d_g[0, i]]
-            q = OP.softmax_t(z_o[0, i], 1.0)[d_g[0, i]]
-            u = uniform01(raw_words(seed, STREAM_ACCEPT, step, 0, i, np.zeros(1, np.uint64)))[0]
-            if abs(u - p / q) > 1e-3:
-                assert (u * q < p) == (i < a_g), (step, i)
-                checked += 1
-        em = [int(x) for x in out["emitted"][0].cpu().numpy()[: a_g + 1]]
-        slots, _ = P.oracle.commit([a_g], [em if len(em) == a_g + 1 else em + [0] * (a_g + 1 - len(em))])
-        assert np.array_equal(out["kv_slots"][0].cpu().numpy()[: a_g + 1], slots[0][: a_g + 1])
+    while not P.oracle.all_done() and step < 60:
+        sampling_step(P, step, seed)
         step += 1
-    assert checked > 0
+    assert P.oracle.all_done()
+    st = P.stats
+    print("stats", st)
+    assert st["decisions_checked"] > 0
+    # draft candidates, first tokens and bonus draws: nearly all have clear margins
+    assert st["sampled_exact"] >= 0.9 * st["sampled_checked"]
     assert P.eng.last_status() == 0
 
 
 def test_sampling_full_width_8b_two_layers():
     """The sampling configuration (8b_sample: T = 1, K = 6) at full width with
-    two layers per model, 64-token prompt: logits within tolerance, accept
-    decisions equal wherever |u - p/q| > 1e-3, KV slots equal."""
+    two layers per model, 64-token prompt: logits within tolerance; sampled
+    candidates, first token, decisions and bonus draws as in the tiny test;
+    KV slots equal."""
     wl = S.WORKLOADS["8b_sample"].replace(target=S.TARGET_8B.replace(n_layers=2),
-                                          draft=S.DRAFT_1B.replace(n_layers=2), prompt_len=64, n_new=16)
+                                          draft=S.DRAFT_1B.replace(n_layers=2), prompt_len=64, n_new=24)
     P = Pair(wl, prefill_chunk=64)
     seed = 5
     P.prefill(seed)
-    K = wl.K
-    checked = 0
-    for step in range(1, 4):
-        out = P.eng.alloc_step_outputs(want_logits=True)
-        P.eng.draft(out, True, 1.0, seed, step)
-        d_g = out["draft"].cpu().numpy()
-        z_g = out["draft_logits"].cpu().numpy()
-        d_o, z_o = P.oracle.draft(step, seed)
-        assert np.abs(z_g - z_o).max() <= LOGIT_TOL
-        P.eng.verify(out, None, 1.0)
-        y_g = out["logits"].cpu().numpy()
-        y_o = P.oracle.verify(d_g)
-        assert np.abs(y_g - y_o).max() <= LOGIT_TOL
-        P.eng.accept_commit(out, True, 1.0, seed, step)
-        a_g = int(out["accept_len"][0])
-        for i in range(min(a_g + 1, K)):
-            p = OP.softmax_t(y_o[0, i], 1.0)[d_g[0, i]]
-            q = OP.softmax_t(z_o[0, i], 1.0)[d_g[0, i]]
-            u = uniform01(raw_words(seed, STREAM_ACCEPT, step, 0, i, np.zeros(1, np.uint64)))[0]
-            if abs(u - p / q) > 1e-3:
-                assert (u * q < p) == (i < a_g), (step, i)
-                checked += 1
-        em = [int(x) for x in out["emitted"][0].cpu().numpy()[: a_g + 1]]
-        slots, _ = P.oracle.commit([a_g], [em if len(em) == a_g + 1 else em + [0] * (a_g + 1 - len(em))])
-        assert np.array_equal(out["kv_slots"][0].cpu().numpy()[: a_g + 1], slots[0][: a_g + 1])
-    assert checked > 0
+    for step in range(1, 5):
+        sampling_step(P, step, seed)
+    st = P.stats
+    print("stats", st)
+    assert st["sampled_exact"] >= 0.9 * st["sampled_checked"]
     assert P.eng.last_status() == 0
+
+
+@pytest.mark.parametrize("vocab", [2048, 128256])
+def test_draft_sampler_on_identical_logits(vocab):
+    """Level 1 for the draft's candidate selection (Eq. 6, sampled at
+    temperature T, and greedy): given draft logits go through the same tile
+    statistics and selection kernel as the LM head's, and the candidates
+    equal the oracle's Gumbel-max (or argmax) winners on the same Philox
+    stream exactly, except where the winner's lead is a few fp32 ulps."""
+    import torch
+    wl = S.WORKLOADS["tiny"].replace(batch=3, K=6, n_new=100, prompt_len=20)
+    if vocab != wl.target.vocab:
+        wl = wl.replace(target=wl.target.replace(vocab=vocab, mask_id=vocab - 1),
+                        draft=wl.draft.replace(vocab=vocab, mask_id=vocab - 1))
+    P = Pair(wl)
+    P.prefill()
+    B, K, V = wl.batch, wl.K, vocab
+    rng = np.random.default_rng(vocab)
+    near = exact = 0
+    for trial in range(12):
+        T = (0.7, 1.0, 1.3)[trial % 3]
+        sample = trial % 4 != 3
+        z = (rng.standard_normal((B, K, V)) * 2.0).astype(np.float32)
+        out = P.eng.alloc_step_outputs()
+        seed, step = 31 + trial, 200 + trial
+        P.eng.set_draft_logits(torch.as_tensor(z, device="cuda"), out, sample, T, seed, step)
+        d_g = out["draft"].cpu().numpy()
+        for b in range(B):
+            d_o = OP.draft_tokens(z[b], sample, T, seed, step, b)
+            for i in range(K):
+                if int(d_g[b, i]) == d_o[i]:
+                    exact += 1
+                    continue
+                sc = (gumbel_scores(z[b, i], T, seed, STREAM_DRAFT, step, b, i) if sample
+                      else z[b, i].astype(np.float32))
+                assert margin(sc) <= GUMBEL_EPS, (trial, b, i, int(d_g[b, i]), d_o[i], margin(sc))
+                near += 1
+    print("exact", exact, "near ties", near)
+    assert near <= 2 and exact >= B * K * 12 - 2
 
 
 def test_weight_packing_round_trip_restores_every_matrix():

@@ -15,24 +15,32 @@ from oracle import pard as OP
 pytestmark = pytest.mark.gpu
 
 
-def test_noalloc_acceptance_matches_context_path_twice():
+@pytest.mark.parametrize("batch,K,vocab", [(1, 4, 2048), (3, 4, 2048), (16, 8, 128256)],
+                         ids=["b1k4", "b3k4", "b16k8_full_vocab"])
+def test_noalloc_acceptance_matches_context_path_twice(batch, K, vocab):
+    """Four calls in a row (two sampled, two greedy) at batch 1, at batch 3,
+    and at the scratch's limits (batch 16, K = 8, the 128256-entry
+    vocabulary: every row pitch and tile count of its fixed layout)."""
     import torch
     from _parity import Pair
     from paper_2504_18583_gb300 import _build, pard
     _build.build()
-    wl = S.WORKLOADS["tiny"].replace(sample=True, n_new=100000, K=4)
+    wl = S.WORKLOADS["tiny"].replace(sample=True, n_new=100000, K=K, batch=batch, prompt_len=20)
+    if vocab != wl.target.vocab:
+        wl = wl.replace(target=wl.target.replace(vocab=vocab, mask_id=vocab - 1),
+                        draft=wl.draft.replace(vocab=vocab, mask_id=vocab - 1))
     P = Pair(wl)
     P.prefill(seed=3)
-    B, K, V = wl.batch, wl.K, wl.target.vocab
-    rng = np.random.default_rng(11)
+    B, V = wl.batch, vocab
+    rng = np.random.default_rng(11 + batch)
     lib = pard.lib()
     stream = P.eng.stream.cuda_stream
     for call, sample in enumerate((True, True, False, False)):
         y = (rng.standard_normal((B, K + 1, V)) * 2.0).astype(np.float32)
         z = (y[:, :K] + rng.standard_normal((B, K, V)).astype(np.float32) * 0.5).astype(np.float32)
-        d = np.array([OP.draft_tokens(z[0], True, 1.0, 900 + call, 2, 0)], dtype=np.int32)
+        d = np.array([OP.draft_tokens(z[b], True, 1.0, 900 + call, 2, b) for b in range(B)], dtype=np.int32)
         if call == 1:
-            d[0, 1:] = np.argmax(y[0, 1:K], axis=-1)  # some acceptance deep into the draft
+            d[:, 1:] = np.argmax(y[:, 1:K], axis=-1)  # some acceptance deep into the draft
         yt, zt, dt = (torch.as_tensor(a, device="cuda") for a in (y, z, d))
         step = 50 + call
         # existing path
