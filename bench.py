@@ -46,6 +46,9 @@ WORKLOAD_DESCS = {
     "8b_sample": WORKLOAD_DESC.replace("512-token prompt, K=8, greedy", "1024-token prompt, K=6, speculative sampling T=1"),
     "8b_batch16": WORKLOAD_DESC.replace("batch 1, 512-token prompt, K=8, greedy, 256 new tokens",
                                         "batch 16, ragged prompts U[128, 2048], K=6, greedy, 128 new tokens"),
+    "70b_greedy": ("70B-shaped target (80 layers, d 8192, 64q/8kv heads, ffn 28672, vocab 128256; 141 GB of bf16 "
+                   "weights) + LLaMA3.2-1B-shaped PARD draft, batch 1, 4096-token context, K=8, greedy, "
+                   "128 new tokens, KV page 16"),
 }
 
 
@@ -237,6 +240,121 @@ def run_reference(args):
     return 0
 
 
+def timed_generation(eng, wl, prompts, timed_steps: int, warmup: int, phase_events: bool, ws: int, seed: int = 1):
+    """Prefill, `warmup` untimed steps, then `timed_steps` decode steps timed
+    with CUDA events on the engine's stream (barrier + synchronize on both
+    sides).  Returns (ms, tokens emitted, kernel launches, per-phase ms lists)."""
+    import torch
+    sample, temp = wl.sample, wl.temperature
+    stream = eng.stream
+    eng.prefill(prompts, wl.n_new, wl.K, sample, temp, seed)
+    out = eng.alloc_step_outputs()
+    for s in range(1, warmup + 1):
+        eng.step(out, sample, temp, seed, step=s)
+    torch.cuda.synchronize()
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    ph = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(timed_steps)]
+    n_emit = torch.zeros((timed_steps, wl.batch), dtype=torch.int32, device="cuda")
+    launches = 0
+    ev[0].record(stream)
+    for i in range(timed_steps):
+        s = warmup + 1 + i
+        if phase_events:
+            ph[i][0].record(stream)
+        eng.draft(out, sample, temp, seed, s)
+        launches += eng.launch_count()
+        if phase_events:
+            ph[i][1].record(stream)
+        eng.verify(out, None, temp)
+        launches += eng.launch_count()
+        if phase_events:
+            ph[i][2].record(stream)
+        eng.accept_commit(out, sample, temp, seed, s)
+        launches += eng.launch_count()
+        if phase_events:
+            ph[i][3].record(stream)
+        n_emit[i].copy_(out["n_emit"])
+    ev[1].record(stream)
+    torch.cuda.synchronize()
+    if ws > 1:
+        torch.distributed.barrier()
+    ms = ev[0].elapsed_time(ev[1])
+    phases = None
+    if phase_events:
+        phases = {k: [ph[i][j].elapsed_time(ph[i][j + 1]) for i in range(timed_steps)]
+                  for j, k in enumerate(("draft", "verify", "accept"))}
+    return ms, int(n_emit.sum().item()), launches, phases
+
+
+def make_engine(wl, host_t=None, host_d=None):
+    """Device weights of the workload (from the host copies when given) and
+    an engine sized for it.  Returns (engine, target weights, draft weights,
+    prompts, seconds spent generating weights)."""
+    import synthetic as S
+    from paper_2504_18583_gb300 import pard
+    t_gen = time.perf_counter()
+    tw = S.device_weights(wl.target, wl.seed, S.TARGET, host=host_t)
+    dw = S.device_weights(wl.draft, wl.seed, S.DRAFT, host=host_d)
+    t_gen = time.perf_counter() - t_gen
+    prompts = [p.tolist() for p in wl.prompts()]
+    max_ctx = max(len(p) for p in prompts) + wl.n_new + 2 * wl.K + 16
+    eng = pard.PardEngine(wl.target, tw, wl.draft, dw, max_batch=wl.batch, max_k=wl.K, max_ctx=max_ctx,
+                          n_pages=wl.n_pages(), prefill_chunk=512, page_order_target=wl.page_order(S.TARGET),
+                          page_order_draft=wl.page_order(S.DRAFT))
+    return eng, tw, dw, prompts, t_gen
+
+
+def step_summary(wl, prompts, ms, toks, phases, steps, warmup, peak):
+    """Tokens/s, per-phase medians and the verify / draft pass rooflines of
+    one timed generation (mean context over the timed steps, summed over the
+    batch; random-init drafts accept ~nothing, so each step adds one token
+    per sequence)."""
+    ver_ms = statistics.median(phases["verify"])
+    dr_ms = statistics.median(phases["draft"])
+    acc_ms = statistics.median(phases["accept"])
+    ctx_mid = sum(len(p) for p in prompts) + wl.batch * (warmup + steps / 2.0)
+    vb = verify_bytes(wl, ctx_mid)
+    db = draft_bytes(wl, ctx_mid)
+    ver_gbs = vb / (ver_ms / 1e3) / 1e9
+    dr_gbs = db / (dr_ms / 1e3) / 1e9
+    return {"value": toks / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms / steps, "steps": steps,
+            "warmup": warmup, "phases_ms": {"draft": dr_ms, "verify": ver_ms, "accept": acc_ms},
+            "verify_roofline": {"bound": "hbm", "achieved": ver_gbs, "peak": peak, "unit": "GB/s",
+                                "frac": ver_gbs / peak, "bytes": vb},
+            "draft_roofline": {"achieved": dr_gbs, "frac": dr_gbs / peak, "bytes": db}}
+
+
+def config_run(name: str, args, ws: int, local: int, peak: float):
+    """One more configuration of the same decode step, timed like the
+    headline (its own seeded weights, prompts, K, batch and sampling)."""
+    import gc
+    import torch
+    import synthetic as S
+    wl = S.WORKLOADS[name]
+    steps = min(args.steps, wl.n_new - 2 - args.warmup)
+    eng, tw, dw, prompts, t_gen = make_engine(wl)
+    try:
+        timed_generation(eng, wl, prompts, 2, 3, False, ws)
+        clocks = ClockSampler(local)
+        clocks.start()
+        ms, toks, launches, phases = timed_generation(eng, wl, prompts, steps, args.warmup, True, ws)
+        clk = clocks.stop()
+        flags = eng.last_status()
+    finally:
+        eng.close()
+        del eng, tw, dw
+        gc.collect()
+        torch.cuda.empty_cache()
+    ms_max, tot = aggregate_over_ranks(ms, toks, ws)
+    out = step_summary(wl, prompts, ms_max, tot, phases, steps, args.warmup, peak)
+    out.update({"workload": name + ": " + WORKLOAD_DESCS[name], "batch": wl.batch, "gpu_launches": launches,
+                "clocks": clk, "device_status": flags, "weights_gen_s": t_gen})
+    return out
+
+
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
@@ -254,8 +372,11 @@ def main():
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the planted-acceptance and autoregressive runs (profiling runs: the timed steps "
                          "are then the last launches)")
-    ap.add_argument("--workload", default="8b_greedy", choices=["8b_greedy", "8b_sample", "8b_batch16"],
-                    help="8b_greedy (the headline), 8b_sample (T = 1, K = 6), 8b_batch16 (16 ragged prompts, K = 6)")
+    ap.add_argument("--workload", default="8b_greedy", choices=["8b_greedy", "8b_sample", "8b_batch16", "70b_greedy"],
+                    help="8b_greedy (the headline), 8b_sample (T = 1, K = 6), 8b_batch16 (16 ragged prompts, K = 6), "
+                         "70b_greedy (70B-shaped target, 4096-token context, K = 8)")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the sampling, batch-16 and 70B configurations the headline run also times")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling aid: truncate both models to this many layers (not a bench number)")
     args = ap.parse_args()
@@ -283,70 +404,24 @@ def main():
         wl = wl.replace(batch=args.batch)
     if args.warmup + args.steps > wl.n_new - 2:
         raise SystemExit(f"warmup + steps must stay below the generation length ({wl.n_new})")
-    keep_host = rank == 0 and not args.no_cpu_baseline
-    t_gen = time.perf_counter()
+    # the CPU baseline times the oracle on the headline's models (the 70B one would hold 141 GB of host copies)
+    keep_host = rank == 0 and not args.no_cpu_baseline and args.workload != "70b_greedy"
+    t_host = time.perf_counter()
     host_t = S.model_weights(wl.target, wl.seed, S.TARGET) if keep_host else None
     host_d = S.model_weights(wl.draft, wl.seed, S.DRAFT) if keep_host else None
-    tw = S.device_weights(wl.target, wl.seed, S.TARGET, host=host_t)
-    dw = S.device_weights(wl.draft, wl.seed, S.DRAFT, host=host_d)
-    t_gen = time.perf_counter() - t_gen
-    prompts = [p.tolist() for p in wl.prompts()]
+    t_host = time.perf_counter() - t_host
+    eng, tw, dw, prompts, t_gen = make_engine(wl, host_t, host_d)
+    t_gen += t_host
     lens = [len(p) for p in prompts]
-    max_ctx = max(lens) + wl.n_new + 2 * wl.K + 16
-    eng = pard.PardEngine(wl.target, tw, wl.draft, dw, max_batch=wl.batch, max_k=wl.K, max_ctx=max_ctx,
-                          n_pages=wl.n_pages(), prefill_chunk=512, page_order_target=wl.page_order(S.TARGET),
-                          page_order_draft=wl.page_order(S.DRAFT))
     stream = eng.stream
 
     sample, temp, seed = wl.sample, wl.temperature, 1
 
-    def generation(timed_steps: int, warmup: int, phase_events: bool):
-        eng.prefill(prompts, wl.n_new, wl.K, sample, temp, seed)
-        out = eng.alloc_step_outputs()
-        for s in range(1, warmup + 1):
-            eng.step(out, sample, temp, seed, step=s)
-        torch.cuda.synchronize()
-        if ws > 1:
-            torch.distributed.barrier()
-        torch.cuda.synchronize()
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-        ph = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(timed_steps)]
-        n_emit = torch.zeros((timed_steps, wl.batch), dtype=torch.int32, device="cuda")
-        launches = 0
-        ev[0].record(stream)
-        for i in range(timed_steps):
-            s = warmup + 1 + i
-            if phase_events:
-                ph[i][0].record(stream)
-            eng.draft(out, sample, temp, seed, s)
-            launches += eng.launch_count()
-            if phase_events:
-                ph[i][1].record(stream)
-            eng.verify(out, None, temp)
-            launches += eng.launch_count()
-            if phase_events:
-                ph[i][2].record(stream)
-            eng.accept_commit(out, sample, temp, seed, s)
-            launches += eng.launch_count()
-            if phase_events:
-                ph[i][3].record(stream)
-            n_emit[i].copy_(out["n_emit"])
-        ev[1].record(stream)
-        torch.cuda.synchronize()
-        if ws > 1:
-            torch.distributed.barrier()
-        ms = ev[0].elapsed_time(ev[1])
-        phases = None
-        if phase_events:
-            phases = {k: [ph[i][j].elapsed_time(ph[i][j + 1]) for i in range(timed_steps)]
-                      for j, k in enumerate(("draft", "verify", "accept"))}
-        return ms, int(n_emit.sum().item()), launches, phases
-
     # untimed warm-up generation (JIT, caches)
-    generation(2, 3, False)
+    timed_generation(eng, wl, prompts, 2, 3, False, ws)
     clocks = ClockSampler(local)
     clocks.start()
-    ms, toks, launches, phases = generation(args.steps, args.warmup, True)
+    ms, toks, launches, phases = timed_generation(eng, wl, prompts, args.steps, args.warmup, True, ws)
     clk = clocks.stop()
     n_state = eng.state()[0][0]
     flags = eng.last_status()
@@ -496,15 +571,21 @@ def main():
 
     # roofline of the verify pass
     peak, peak_kind = peaks()
-    ver_ms = statistics.median(phases["verify"])
-    dr_ms = statistics.median(phases["draft"])
-    acc_ms = statistics.median(phases["accept"])
-    # mean context during the timed steps, summed over the batch (a ~ 0 with random-init drafts)
-    ctx_mid = sum(lens) + wl.batch * (args.warmup + args.steps / 2.0)
-    vb = verify_bytes(wl, ctx_mid)
-    db = draft_bytes(wl, ctx_mid)
-    ver_gbs = vb / (ver_ms / 1e3) / 1e9
-    dr_gbs = db / (dr_ms / 1e3) / 1e9
+    summ = step_summary(wl, prompts, ms, toks, phases, args.steps, args.warmup, peak)
+    ver_ms, dr_ms, acc_ms = (summ["phases_ms"][k] for k in ("verify", "draft", "accept"))
+    vb, ver_gbs = summ["verify_roofline"]["bytes"], summ["verify_roofline"]["achieved"]
+    db, dr_gbs = summ["draft_roofline"]["bytes"], summ["draft_roofline"]["achieved"]
+
+    # the other configurations, each on its own seeded weights (the headline's
+    # engine is released first: the 70B-shaped target alone is 141 GB)
+    configs = None
+    if headline and not args.no_configs:
+        import gc
+        eng.close()
+        del eng, tw, dw
+        gc.collect()
+        torch.cuda.empty_cache()
+        configs = {name: config_run(name, args, ws, local, peak) for name in ("8b_sample", "8b_batch16", "70b_greedy")}
 
     cpu = None
     if keep_host and ws == 1:
@@ -537,6 +618,7 @@ def main():
                      "bytes_note": "target weights 15.01 GB + KV read over the context + K+1 rows of KV written"},
         "phases_ms": {"draft": dr_ms, "verify": ver_ms, "accept": acc_ms},
         "draft_roofline": {"achieved": dr_gbs, "frac": dr_gbs / peak, "bytes": db},
+        "configs": configs,
         "planted_acceptance": planted,
         "autoregressive_baseline": ar,
         "vanilla_sd_baseline": vsd,

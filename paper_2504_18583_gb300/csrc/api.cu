@@ -620,6 +620,7 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
     c->st.samp_cnt = c->at<int>(o.st_scnt); c->st.kmax = lim->max_k;
     c->call = c->at<CallArgs>(o.call); c->status = c->at<uint32_t>(o.status);
     c->paths = c->at<uint32_t>(o.paths);
+
     c->tmp_pos = c->at<int>(o.tmp_pos); c->g_plen = c->at<int>(o.g_plen);
     c->mask_ids = c->at<int>(o.mask_ids);
 

@@ -110,6 +110,7 @@ constexpr uint32_t kAttnPathPush = 1u << 0;
 constexpr uint32_t kAttnPathPull = 1u << 1;
 constexpr int kAttnPathSplit0 = 3;
 
+
 // Per-sequence decode state, in the workspace.
 struct DevState {
   int* n;          // [B] tokens so far, the pending one included (target cache holds n-1)

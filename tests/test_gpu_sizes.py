@@ -88,6 +88,8 @@ def test_70b_widths_two_layers_4096_context():
         greedy_step(P, step)
     bits = P.eng.attention_paths()
     print("paths", hex(bits), "cluster sizes", split_sizes(bits), "stats", P.stats)
+    # the 9 verify rows are two row blocks of 8 at group 8; 16-CTA clusters
+    assert split_sizes(bits) == [16]
     assert P.eng.last_status() == 0
 
 
