@@ -217,19 +217,24 @@ def greedy_step(P: Pair, step: int, inject=None, sequential: bool = False):
     return dict(a=a_gpu, emitted=em_gpu, slots=slots_gpu, d=d_gpu, y=y_gpu, z=z_gpu)
 
 
-def sampling_step(P: Pair, step: int, seed: int) -> dict:
+def sampling_step(P: Pair, step: int, seed: int, sequential: bool = False) -> dict:
     """One teacher-forced speculative-sampling step (Section 2.2 with the
-    draft of Eq. 6 at temperature T): draft logits, verify logits within
-    LOGIT_TOL; the draft's Gumbel-max candidates, the accept / reject
-    decisions and the bonus draw against the oracle's on the same Philox
-    streams wherever the margins are clear; KV slots bit-exact.  The oracle
-    is then committed with the GPU's tokens."""
+    draft of Eq. 6 at temperature T; sequential: vanilla speculative
+    decoding's K-pass draft, the oracle fed the GPU's candidates between
+    passes): draft logits, verify logits within LOGIT_TOL; the draft's
+    Gumbel-max candidates, the accept / reject decisions and the bonus draw
+    against the oracle's on the same Philox streams wherever the margins are
+    clear; KV slots bit-exact.  The oracle is then committed with the GPU's
+    tokens."""
     wl, K, T = P.wl, P.wl.K, P.wl.temperature
     out = P.eng.alloc_step_outputs(want_logits=True)
-    P.eng.draft(out, True, T, seed, step)
+    if sequential:
+        P.eng.draft_sequential(out, True, T, seed, step)
+    else:
+        P.eng.draft(out, True, T, seed, step)
     d_g = out["draft"].cpu().numpy()
     z_g = out["draft_logits"].cpu().numpy()
-    d_o, z_o = P.oracle.draft(step, seed)
+    d_o, z_o = P.oracle.draft_sequential(step, seed, feed=d_g) if sequential else P.oracle.draft(step, seed)
     for b in P.active():
         for i in range(K):
             err = float(np.abs(z_g[b, i] - z_o[b, i]).max())

@@ -379,6 +379,27 @@ def test_sampling_full_width_8b_two_layers():
     assert P.eng.last_status() == 0
 
 
+def test_vanilla_sd_sampled_sequential_draft():
+    """The sampled form of vanilla speculative decoding's drafting stage
+    (Section 2.2): every draft pass draws its candidate by Gumbel-max from
+    its own logits (Philox stream 0, row i); candidates, decisions and bonus
+    draws against the oracle's sequential draft fed the GPU's candidates,
+    margins as in the other sampling tests; batch 2, ragged prompts."""
+    wl = S.WORKLOADS["tiny"].replace(sample=True, n_new=30, batch=2, prompt_len=None, prompt_len_range=(20, 45))
+    P = Pair(wl)
+    seed = 13
+    P.prefill(seed)
+    step = 1
+    while not P.oracle.all_done() and step < 40:
+        sampling_step(P, step, seed, sequential=True)
+        step += 1
+    st = P.stats
+    print("stats", st)
+    assert P.oracle.all_done()
+    assert st["sampled_exact"] >= 0.9 * st["sampled_checked"]
+    assert P.eng.last_status() == 0
+
+
 @pytest.mark.parametrize("vocab", [2048, 128256])
 def test_draft_sampler_on_identical_logits(vocab):
     """Level 1 for the draft's candidate selection (Eq. 6, sampled at
