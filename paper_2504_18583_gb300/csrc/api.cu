@@ -102,8 +102,11 @@ int round_up(int x, int m) { return (x + m - 1) / m * m; }
 Dims make_dims(const pard_model_cfg& t, const pard_model_cfg& d, const pard_limits& lim, int sm) {
   Dims D;
   D.m_dec = lim.max_batch * 2 * lim.max_k;
-  D.MC = round_up(std::max(D.m_dec, lim.prefill_chunk), 64);
-  D.gcap = lim.max_batch <= 16 ? 16 : round_up(lim.max_batch, 64);  // whole token tiles of the LM-head input
+  // whole token tiles of the widest pass (tiles of 128 rows above 64)
+  const int mrows = std::max(D.m_dec, lim.prefill_chunk);
+  D.MC = round_up(mrows, mrows > 64 ? 128 : 64);
+  // whole token tiles of the LM-head input
+  D.gcap = lim.max_batch <= 16 ? 16 : (lim.max_batch <= 64 ? 64 : round_up(lim.max_batch, 128));
   D.dmax = std::max(t.d_model, d.d_model);
   D.qdmax = std::max(t.n_q_heads * t.head_dim, d.n_q_heads * d.head_dim);
   D.ffnmax = std::max(t.ffn, d.ffn);
@@ -140,7 +143,7 @@ WsOffsets layout_ws(const Dims& D, const pard_limits& lim) {
   o.ssq = L.take((size_t)(D.dmax / 128) * D.MC * 4);
   o.ssqg = L.take((size_t)(D.dmax / 128) * D.MC * 4);
   o.q = L.take((size_t)D.MC * D.qdmax * 4);
-  o.gpart = L.take((size_t)D.sm * 2 * kTileN * 64 * 4);
+  o.gpart = L.take((size_t)D.sm * 2 * kTileN * (D.MC > 64 ? 128 : 64) * 4);  // two partial tiles per CTA
   o.gcnt = L.take((size_t)65536 * 4);
   o.stats_t = L.take((size_t)D.w_tiles * D.MC * 16);
   o.stats_it = L.take((size_t)D.w_tiles * D.MC * 8);
@@ -249,7 +252,9 @@ CUtensorMap make_map(const void* base, int rows, int cols, int box_rows) {
   return m;
 }
 
-int pick_tt(int rows) { return rows <= 16 ? 16 : 64; }
+// Token tile of a pass of up to `rows` rows: 16, 64, or 128 (65 and more
+// rows: one pass over the weights covers 128 of them).
+int pick_tt(int rows) { return rows <= 16 ? 16 : (rows <= 64 ? 64 : 128); }
 
 }  // namespace
 
@@ -280,6 +285,7 @@ struct pard_ctx {
   // host state
   std::vector<int> order[2];
   int batch = 0, K = 0, n_new = 0;
+  std::vector<int> ctx_est;  // per sequence: prompt + n_new, an upper bound of its context (attention splits)
   bool prefilled = false;
   bool last_draft_sampled = false;
   bool unpacked = false;
@@ -302,6 +308,7 @@ GemmArgs gemm_base(pard_ctx* c, int rows_cap, int tt) {
   GemmArgs a;
   std::memset(&a, 0, sizeof(a));
   a.tok_tiles = (rows_cap + tt - 1) / tt;
+  a.n_tok = a.tok_tiles == 1 ? round_up(rows_cap, 8) : 0;
   a.m_cap = c->D.MC;
   a.m_dev = c->rp.m_dev;
   a.partials = c->gpart;
@@ -335,6 +342,21 @@ AttnGeom attn_geometry(pard_ctx* c, int mi, int rows_per_seq, int batch) {
   g.groups = batch * cf.n_kv_heads * g.row_blocks;
   const int n_kt = (c->lim.max_ctx + 31) / 32;  // 32-key chunks at the longest context
   g.n_split = std::max(1, std::min({c->attn_split_cap, n_kt, (2 * c->sm + g.groups - 1) / g.groups}));
+  if (batch > 1 && (int)c->ctx_est.size() >= batch) {
+    // Ragged contexts: the kernel lasts as long as the longest sequence's
+    // units, which walk its chunks / n_split each.  Split until that share is
+    // no longer than the average CTA's share of all units' chunks at two
+    // CTAs per SM (more splits only add per-CTA start-up and combine work).
+    long total = 0, longest = 0;
+    for (int b = 0; b < batch; ++b) {
+      const long ch = (c->ctx_est[b] + 31) / 32;
+      total += ch;
+      longest = std::max(longest, ch);
+    }
+    total *= (long)cf.n_kv_heads * g.row_blocks;
+    const long bal = total > 0 ? (longest * 2 * c->sm + total - 1) / total : 1;
+    g.n_split = std::max<long>(g.n_split, std::min<long>({bal, (long)c->attn_split_cap, (long)n_kt}));
+  }
   return g;
 }
 
@@ -343,7 +365,7 @@ struct LayerPlan {
   GemmArgs qkv, o, gu, dn;
   AttnArgs at;
 };
-LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch, const int* pt_attn,
+LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int tt_gu, int batch, const int* pt_attn,
                      const AttnGeom& geo, int fixed_rows) {
   Model& M = c->m[mi];
   const pard_model_cfg& cf = M.cfg;
@@ -386,6 +408,7 @@ LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch
     a.batch = batch; a.hq = cf.n_q_heads; a.hkv = cf.n_kv_heads; a.hd = cf.head_dim;
     a.page_size = c->lim.page_size; a.n_pages = c->lim.n_pages;
     a.row_blocks = geo.row_blocks; a.n_split = geo.n_split;
+    a.nbuf = (long)geo.groups * geo.n_split > 2L * c->sm ? 2 : 4;
     a.scale = (float)(1.0 / std::sqrt((double)cf.head_dim));
     a.x_out = c->xo; a.x_rows = 2 * c->D.MC;
     a.status = c->status;
@@ -408,7 +431,7 @@ LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch
   // RMSNorm -> gate/up (paired 64-row tiles) -> SiLU(gate) * up
   {
     GemmArgs& a = P.gu;
-    a = gemm_base(c, rows_cap, tt);
+    a = gemm_base(c, rows_cap, tt_gu);
     a.wmap[0] = Mp.g; a.wmap[1] = Mp.u;
     a.wpk[0] = M.P[l].t[W_G]; a.wpk[1] = M.P[l].t[W_U];
     if (!a.wpk[0] || !a.wpk[1]) a.wpk[0] = a.wpk[1] = nullptr;
@@ -445,15 +468,25 @@ LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int batch
 // by its sequence index.
 void run_layers(pard_ctx* c, int mi, int rows_cap, int batch, int rows_per_seq, const int* pt_attn,
                 cudaStream_t s, int fixed_rows = 0) {
-  const int tt = pick_tt(rows_cap);
+  // Above 64 rows the gate/up projection takes the 128-token tile (one pass
+  // over its weights for all rows), the QKV, O and down projections keep
+  // 64-token tiles (two passes): they have only 32-48 output tiles, so with
+  // 128-token tiles each tile's split-K finish and epilogue (8 chunks) falls
+  // on few CTAs and outlasts the bytes saved.
+  const int tt_gu = pick_tt(rows_cap);
+  const int tt = std::min(tt_gu, 64);
   const AttnGeom geo = attn_geometry(c, mi, rows_per_seq, batch);
   for (int l = 0; l < c->m[mi].cfg.n_layers; ++l) {
-    LayerPlan P = layer_plan(c, mi, l, rows_cap, tt, batch, pt_attn, geo, fixed_rows);
+    LayerPlan P = layer_plan(c, mi, l, rows_cap, tt, tt_gu, batch, pt_attn, geo, fixed_rows);
+    // the pass's row count is written by the embedding kernel, which directly
+    // precedes only the first QKV projection
+    P.qkv.m_early = l > 0;
+    P.o.m_early = P.gu.m_early = P.dn.m_early = 1;
     run_gemm(c, P.qkv, tt, s);
     launch_attention(P.at, geo.groups * geo.n_split, s, true);
     c->launches++;
     run_gemm(c, P.o, tt, s);
-    run_gemm(c, P.gu, tt, s);
+    run_gemm(c, P.gu, tt_gu, s);
     run_gemm(c, P.dn, tt, s);
   }
 }
@@ -476,6 +509,7 @@ GemmArgs lm_args(pard_ctx* c, int mi, const __nv_bfloat16* x, int x_rows, const 
   a.ssq_in = ssq_in; a.ssq_tiles = M.cfg.d_model / 128; a.inv_d = 1.0f / M.cfg.d_model; a.eps = M.cfg.rms_eps;
   a.logits = logits; a.row_out = row_out; a.row_gi = row_gi; a.row_seq = row_seq;
   a.stats = stats; a.stats_i = stats_i; a.vocab = M.cfg.vocab; a.gumbel_stream = gumbel_stream;
+  a.m_early = 1;  // the LM head follows the whole layer stack (or the prefill's gather), far from its row count's writer
   return a;
 }
 
@@ -763,6 +797,8 @@ pard_status pard_prefill(pard_ctx* c, const int32_t* d_tokens, const int32_t* h_
     c->batch = batch;
     c->K = K;
     c->n_new = n_new;
+    c->ctx_est.assign(batch, 0);
+    for (int b = 0; b < batch; ++b) c->ctx_est[b] = h_lens[b] + n_new;
     c->prefilled = false;
     set_call(c, seed, 0, temperature, sample, s);
     const int chunk = c->lim.prefill_chunk;

@@ -20,11 +20,14 @@
 
 namespace pard {
 
-constexpr int kAttnBufs = 4;  // K/V chunk ring of the standalone kernel (3 chunks in flight)
-
-template <int HD, int GROUP>
+// K/V chunk ring: NBUF = 4 buffers (three chunks in flight, ~87 KB at
+// hd = 128, two CTAs per SM) when a pass has few units, as at batch 1; NBUF =
+// 2 (one chunk in flight, four CTAs per SM) when its units fill the SMs more
+// than twice over (ragged batches with long contexts), where the latency of
+// a unit's dependent steps is hidden by the other CTAs' warps instead.
+template <int HD, int GROUP, int NBUF>
 __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constant__ AttnArgs a) {
-  using C = AttnCfg<HD, kAttnBufs>;
+  using C = AttnCfg<HD, NBUF>;
   constexpr int LD = C::kPartLd;
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_pos[kMaxQV];
@@ -49,7 +52,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
   // had itself waited for them before it let this grid start: the unit reads
   // them before waiting, and Q after.
   const int M = a.rows_per_seq > 0 ? a.batch * a.rows_per_seq : __ldcg(a.m_dev);
-  const AttnRows R = attn_unit<HD, GROUP, kAttnBufs>(a, b, kvh, rb, (int)rank, (int)NS, M, smem, s_pos,
+  const AttnRows R = attn_unit<HD, GROUP, NBUF>(a, b, kvh, rb, (int)rank, (int)NS, M, smem, s_pos,
                                                      threadIdx.x, [] { __syncthreads(); }, [] { pdl_wait(); });
   const int row0 = R.row0, nqv = R.nrows * GROUP;
   // the next kernel may start streaming its weights once the key/value reads
@@ -72,7 +75,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
   const uint32_t recv_bytes = NS * (uint32_t)cnt * LD * 4;
   const bool push = NS > 1 && recv_off + recv_bytes <= (uint32_t)C::kKV;
   if (a.paths && rank == 0 && threadIdx.x == 0)
-    atomicOr(a.paths, (NS == 1 ? 0u : push ? kAttnPathPush : kAttnPathPull) | (1u << (kAttnPathSplit0 + NS)));
+    atomicOr(a.paths, (NS == 1 ? 0u : push ? kAttnPathPush : kAttnPathPull) | (NBUF == 2 ? kAttnPathRing2 : 0u) |
+                          (1u << (kAttnPathSplit0 + NS)));
   // every thread's partial writes, ordered before the async-proxy reads of
   // the bulk copies below, and every warp's partial in shared memory
   fence_proxy_async_smem();
@@ -180,14 +184,14 @@ __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const __grid_constan
   cluster_sync();  // peers may still be reading this CTA's partial
 }
 
-template <int HD, int GROUP>
-static cudaError_t launch_attn_t(const AttnArgs& a, int grid, int cluster, cudaStream_t s, bool pdl) {
+template <int HD, int GROUP, int NBUF>
+static cudaError_t launch_attn_nb(const AttnArgs& a, int grid, int cluster, cudaStream_t s, bool pdl) {
   static bool configured = false;
-  const int smem = AttnCfg<HD, kAttnBufs>::kSmem;
+  const int smem = AttnCfg<HD, NBUF>::kSmem;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD, GROUP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD, GROUP, NBUF>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(attn_kernel<HD, GROUP>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    e = cudaFuncSetAttribute(attn_kernel<HD, GROUP, NBUF>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     configured = true;
   }
@@ -205,7 +209,13 @@ static cudaError_t launch_attn_t(const AttnArgs& a, int grid, int cluster, cudaS
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, attn_kernel<HD, GROUP>, a);
+  return cudaLaunchKernelEx(&cfg, attn_kernel<HD, GROUP, NBUF>, a);
+}
+
+template <int HD, int GROUP>
+static cudaError_t launch_attn_t(const AttnArgs& a, int grid, int cluster, cudaStream_t s, bool pdl) {
+  return a.nbuf == 2 ? launch_attn_nb<HD, GROUP, 2>(a, grid, cluster, s, pdl)
+                     : launch_attn_nb<HD, GROUP, 4>(a, grid, cluster, s, pdl);
 }
 
 int attention_rows_per_block(int group) { return kMaxQV / group; }

@@ -190,6 +190,115 @@ struct AttnRows {
   int n_chunks;  // 32-key chunks of the unit's key range (all splits)
 };
 
+// A unit whose query vectors fit in two warps and which walks at least this
+// many chunks splits every chunk's keys between two warp pairs (see attn_unit).
+constexpr int kKeyHalvesMinChunks = 3;
+
+// Online-softmax attention of one warp's 16 query vectors (rows qa = 16 q +
+// g and qb = qa + 8 of the lane's quad g) over keys koff .. koff + 8 NJG - 1
+// of the chunk ch landed in sK / sV (fp16): S = Q K^T on NJG 8-key n-tiles,
+// scale and causal mask (key position <= row position), running max / sum
+// update with the rescale of o, then O += P V with P as the A fragments.
+template <int HD, int NJG, int ROWB>
+__device__ __forceinline__ void attn_chunk(const uint8_t* sK, const uint8_t* sV, int koff, int ch, uint32_t q_base,
+                                           int posa, int posb, float scale, float (&o)[HD / 8][4], float& ma,
+                                           float& mb, float& la, float& lb, int lane) {
+  constexpr int KS = HD / 16;
+  constexpr int NT = HD / 8;
+  const int g = lane >> 2, c4 = lane & 3;
+  // NACC accumulator sets over alternate k-steps keep four independent MMA
+  // chains in flight when the warp covers only NJG = 2 n-tiles
+  constexpr int NACC = NJG >= 4 ? 1 : 4 / NJG;
+  float sacc[NACC][NJG][4];
+#pragma unroll
+  for (int r = 0; r < NACC; ++r)
+#pragma unroll
+    for (int j = 0; j < NJG; ++j) sacc[r][j][0] = sacc[r][j][1] = sacc[r][j][2] = sacc[r][j][3] = 0.f;
+#pragma unroll
+  for (int ks = 0; ks < KS; ++ks) {
+    uint32_t qf[4], kb[NJG][2];
+    ldsm_x4(qf, q_base + ks * 32);
+#pragma unroll
+    for (int j = 0; j < NJG; ++j) {
+      const uint8_t* krow = sK + (koff + j * 8 + g) * ROWB;
+      kb[j][0] = *reinterpret_cast<const uint32_t*>(krow + (ks * 16 + 2 * c4) * 2);
+      kb[j][1] = *reinterpret_cast<const uint32_t*>(krow + (ks * 16 + 8 + 2 * c4) * 2);
+    }
+    // independent accumulators back to back
+#pragma unroll
+    for (int j = 0; j < NJG; ++j) mma_f16_16816(sacc[ks % NACC][j], qf, kb[j][0], kb[j][1]);
+  }
+  float s[NJG][4];
+#pragma unroll
+  for (int j = 0; j < NJG; ++j)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      float v = sacc[0][j][e];
+#pragma unroll
+      for (int r = 1; r < NACC; ++r) v += sacc[r][j][e];
+      s[j][e] = v;
+    }
+  // scale, causal mask, online softmax (rows qa and qb)
+  float mxa = -INFINITY, mxb = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < NJG; ++j) {
+    const int kp = ch * kKeyChunk + koff + j * 8 + 2 * c4;
+    s[j][0] = kp <= posa ? s[j][0] * scale : -INFINITY;
+    s[j][1] = kp + 1 <= posa ? s[j][1] * scale : -INFINITY;
+    s[j][2] = kp <= posb ? s[j][2] * scale : -INFINITY;
+    s[j][3] = kp + 1 <= posb ? s[j][3] * scale : -INFINITY;
+    mxa = fmaxf(mxa, fmaxf(s[j][0], s[j][1]));
+    mxb = fmaxf(mxb, fmaxf(s[j][2], s[j][3]));
+  }
+  mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, 1));
+  mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, 2));
+  mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, 1));
+  mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, 2));
+  const float mna = fmaxf(ma, mxa), mnb = fmaxf(mb, mxb);
+  const float ca = mna == -INFINITY ? 1.f : expf(ma - mna);
+  const float cb = mnb == -INFINITY ? 1.f : expf(mb - mnb);
+  float sa = 0.f, sb = 0.f;
+#pragma unroll
+  for (int j = 0; j < NJG; ++j) {
+    s[j][0] = s[j][0] == -INFINITY ? 0.f : expf(s[j][0] - mna);
+    s[j][1] = s[j][1] == -INFINITY ? 0.f : expf(s[j][1] - mna);
+    s[j][2] = s[j][2] == -INFINITY ? 0.f : expf(s[j][2] - mnb);
+    s[j][3] = s[j][3] == -INFINITY ? 0.f : expf(s[j][3] - mnb);
+    sa += s[j][0] + s[j][1];
+    sb += s[j][2] + s[j][3];
+  }
+  sa += __shfl_xor_sync(0xffffffffu, sa, 1);
+  sa += __shfl_xor_sync(0xffffffffu, sa, 2);
+  sb += __shfl_xor_sync(0xffffffffu, sb, 1);
+  sb += __shfl_xor_sync(0xffffffffu, sb, 2);
+  la = la * ca + sa;
+  lb = lb * cb + sb;
+  ma = mna;
+  mb = mnb;
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    o[nt][0] *= ca; o[nt][1] *= ca; o[nt][2] *= cb; o[nt][3] *= cb;
+  }
+  // O += P V: P as A fragments (keys are the k dimension), V via ldmatrix.trans
+#pragma unroll
+  for (int kk = 0; kk < NJG / 2; ++kk) {
+    uint32_t pf[4];
+    pf[0] = pack_h2(s[2 * kk][0], s[2 * kk][1]);
+    pf[1] = pack_h2(s[2 * kk][2], s[2 * kk][3]);
+    pf[2] = pack_h2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+    pf[3] = pack_h2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+    const uint32_t vrow = smem_u32(sV + (koff + kk * 16 + (lane & 15)) * ROWB);
+#pragma unroll
+    for (int n0 = 0; n0 < NT; n0 += 4) {
+      uint32_t vb[4][2];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) ldsm_x2_trans(vb[u][0], vb[u][1], vrow + (n0 + u) * 16);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) mma_f16_16816(o[n0 + u], pf, vb[u][0], vb[u][1]);
+    }
+  }
+}
+
 // One attention work unit of 4 warps (tid 0..127, warp = tid / 32): sequence
 // b, kv head kvh, row block rb (rows row0 .. row0 + nrows - 1 of the pass,
 // query vectors qv = r * GROUP + head), key split sp of ns over the 32-key
@@ -212,7 +321,6 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
   static_assert(NBUF >= 2 && NBUF <= 4, "chunk ring of 2 to 4 buffers");
   using C = AttnCfg<HD, NBUF>;
   constexpr int RB = kMaxQV / GROUP;  // rows per block
-  constexpr int KS = HD / 16;
   constexpr int NT = HD / 8;
   constexpr int NJ = kKeyChunk / 8;  // 8-key n-tiles per chunk
   const int warp = tid >> 5, lane = tid & 31;
@@ -295,7 +403,15 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
     }
   }
   bar();
-  const int qa = warp * 16 + g, qb = qa + 8;
+  // Warp roles.  Query vectors are tiled 16 to a warp.  When they fit in two
+  // warps and the unit walks at least kKeyHalvesMinChunks chunks, the other
+  // two warps would idle: instead warps 0-1 take keys 0-15 and warps 2-3
+  // keys 16-31 of every chunk, each pair with its own online-softmax state,
+  // and the pairs' states are merged once after the last chunk.
+  const int ng = ((nqv + 15) / 16 <= 2 && n >= kKeyHalvesMinChunks) ? 2 : 1;
+  const int qtile = ng == 2 ? (warp & 1) : warp;
+  const int kgrp = ng == 2 ? (warp >> 1) : 0;
+  const int qa = qtile * 16 + g, qb = qa + 8;
   const int posa = qa < nqv ? s_pos[qa / GROUP] : -1, posb = qb < nqv ? s_pos[qb / GROUP] : -1;
 
   // ---- K/V chunk ring: NBUF - 1 chunks in flight ----
@@ -309,9 +425,9 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
   float ma = -INFINITY, mb = -INFINITY, la = 0.f, lb = 0.f;
-  const bool active = warp * 16 < nqv;
+  const bool active = qtile * 16 < nqv;
   // ldmatrix.x4 row address of this lane in the warp's 16-row Q tile
-  const uint32_t q_base = smem_u32(sQ) + (uint32_t)((warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * C::kRowBytes +
+  const uint32_t q_base = smem_u32(sQ) + (uint32_t)((qtile * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * C::kRowBytes +
                                                     ((lane >> 4) & 1) * 16);
 
   for (int t = 0; t < n; ++t) {
@@ -328,90 +444,62 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
       ++issued;
     }
     if (active) {
-      // S = Q K^T for the chunk's keys: NJ n-tiles of 8 keys, Q fragments per k-step
-      float s[NJ][4];
-#pragma unroll
-      for (int j = 0; j < NJ; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
-#pragma unroll
-      for (int ks = 0; ks < KS; ++ks) {
-        uint32_t qf[4], kb[NJ][2];
-        ldsm_x4(qf, q_base + ks * 32);
-#pragma unroll
-        for (int j = 0; j < NJ; ++j) {
-          const uint8_t* krow = sK + (j * 8 + g) * C::kRowBytes;
-          kb[j][0] = *reinterpret_cast<const uint32_t*>(krow + (ks * 16 + 2 * c4) * 2);
-          kb[j][1] = *reinterpret_cast<const uint32_t*>(krow + (ks * 16 + 8 + 2 * c4) * 2);
-        }
-        // independent accumulators back to back
-#pragma unroll
-        for (int j = 0; j < NJ; ++j) mma_f16_16816(s[j], qf, kb[j][0], kb[j][1]);
-      }
-      // scale, causal mask, online softmax (rows qa and qb)
-      float mxa = -INFINITY, mxb = -INFINITY;
-#pragma unroll
-      for (int j = 0; j < NJ; ++j) {
-        const int kp = ch * kKeyChunk + j * 8 + 2 * c4;
-        s[j][0] = kp <= posa ? s[j][0] * a.scale : -INFINITY;
-        s[j][1] = kp + 1 <= posa ? s[j][1] * a.scale : -INFINITY;
-        s[j][2] = kp <= posb ? s[j][2] * a.scale : -INFINITY;
-        s[j][3] = kp + 1 <= posb ? s[j][3] * a.scale : -INFINITY;
-        mxa = fmaxf(mxa, fmaxf(s[j][0], s[j][1]));
-        mxb = fmaxf(mxb, fmaxf(s[j][2], s[j][3]));
-      }
-      mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, 1));
-      mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, 2));
-      mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, 1));
-      mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, 2));
-      const float mna = fmaxf(ma, mxa), mnb = fmaxf(mb, mxb);
-      const float ca = mna == -INFINITY ? 1.f : expf(ma - mna);
-      const float cb = mnb == -INFINITY ? 1.f : expf(mb - mnb);
-      float sa = 0.f, sb = 0.f;
-#pragma unroll
-      for (int j = 0; j < NJ; ++j) {
-        s[j][0] = s[j][0] == -INFINITY ? 0.f : expf(s[j][0] - mna);
-        s[j][1] = s[j][1] == -INFINITY ? 0.f : expf(s[j][1] - mna);
-        s[j][2] = s[j][2] == -INFINITY ? 0.f : expf(s[j][2] - mnb);
-        s[j][3] = s[j][3] == -INFINITY ? 0.f : expf(s[j][3] - mnb);
-        sa += s[j][0] + s[j][1];
-        sb += s[j][2] + s[j][3];
-      }
-      sa += __shfl_xor_sync(0xffffffffu, sa, 1);
-      sa += __shfl_xor_sync(0xffffffffu, sa, 2);
-      sb += __shfl_xor_sync(0xffffffffu, sb, 1);
-      sb += __shfl_xor_sync(0xffffffffu, sb, 2);
-      la = la * ca + sa;
-      lb = lb * cb + sb;
-      ma = mna;
-      mb = mnb;
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        o[nt][0] *= ca; o[nt][1] *= ca; o[nt][2] *= cb; o[nt][3] *= cb;
-      }
-      // O += P V: P as A fragments (keys are the k dimension), V via ldmatrix.trans
-#pragma unroll
-      for (int kk = 0; kk < NJ / 2; ++kk) {
-        uint32_t pf[4];
-        pf[0] = pack_h2(s[2 * kk][0], s[2 * kk][1]);
-        pf[1] = pack_h2(s[2 * kk][2], s[2 * kk][3]);
-        pf[2] = pack_h2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-        pf[3] = pack_h2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
-        const uint32_t vrow = smem_u32(sV + (kk * 16 + (lane & 15)) * C::kRowBytes);
-#pragma unroll
-        for (int n0 = 0; n0 < NT; n0 += 4) {
-          uint32_t vb[4][2];
-#pragma unroll
-          for (int u = 0; u < 4; ++u) ldsm_x2_trans(vb[u][0], vb[u][1], vrow + (n0 + u) * 16);
-#pragma unroll
-          for (int u = 0; u < 4; ++u) mma_f16_16816(o[n0 + u], pf, vb[u][0], vb[u][1]);
-        }
-      }
+      if (ng == 2)
+        attn_chunk<HD, NJ / 2, C::kRowBytes>(sK, sV, kgrp * (kKeyChunk / 2), ch, q_base, posa, posb, a.scale, o, ma,
+                                             mb, la, lb, lane);
+      else
+        attn_chunk<HD, NJ, C::kRowBytes>(sK, sV, 0, ch, q_base, posa, posb, a.scale, o, ma, mb, la, lb, lane);
     }
   }
   bar();  // K/V and Q buffers are reused for the partial results below
 
-  // partial (unnormalised o, m, l) of this CTA in its own shared memory
   float* part = reinterpret_cast<float*>(smem);
-  if (active) {
+  if (ng == 2) {
+    // Warps 2-3 hand their state to their twins in warps 0-1 (same lane, same
+    // query vectors) through partial rows 32-63, which no push into this
+    // CTA's receive area reaches: a unit walking kKeyHalvesMinChunks chunks
+    // or more keeps the receive area above that many ring buffers.
+    static_assert(2 * kKeyHalvesMinChunks * C::kTileBytes >= kMaxQV * C::kPartLd * 4,
+                  "key-half merge rows overlap the push receive area");
+    float* twin = part + (size_t)(kMaxQV / 2) * C::kPartLd;
+    if (active && kgrp == 1) {
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        const int d = nt * 8 + 2 * c4;
+        *reinterpret_cast<float2*>(twin + qa * C::kPartLd + d) = make_float2(o[nt][0], o[nt][1]);
+        *reinterpret_cast<float2*>(twin + qb * C::kPartLd + d) = make_float2(o[nt][2], o[nt][3]);
+      }
+      if (c4 == 0) {
+        *reinterpret_cast<float2*>(twin + qa * C::kPartLd + HD) = make_float2(ma, la);
+        *reinterpret_cast<float2*>(twin + qb * C::kPartLd + HD) = make_float2(mb, lb);
+      }
+    }
+    bar();
+    if (active && kgrp == 0) {
+      const float2 mla = *reinterpret_cast<const float2*>(twin + qa * C::kPartLd + HD);
+      const float2 mlb = *reinterpret_cast<const float2*>(twin + qb * C::kPartLd + HD);
+      const float na = fmaxf(ma, mla.x), nb = fmaxf(mb, mlb.x);
+      const float sa0 = ma == -INFINITY ? 0.f : expf(ma - na), sa1 = mla.x == -INFINITY ? 0.f : expf(mla.x - na);
+      const float sb0 = mb == -INFINITY ? 0.f : expf(mb - nb), sb1 = mlb.x == -INFINITY ? 0.f : expf(mlb.x - nb);
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        const int d = nt * 8 + 2 * c4;
+        const float2 ta = *reinterpret_cast<const float2*>(twin + qa * C::kPartLd + d);
+        const float2 tb = *reinterpret_cast<const float2*>(twin + qb * C::kPartLd + d);
+        o[nt][0] = o[nt][0] * sa0 + ta.x * sa1;
+        o[nt][1] = o[nt][1] * sa0 + ta.y * sa1;
+        o[nt][2] = o[nt][2] * sb0 + tb.x * sb1;
+        o[nt][3] = o[nt][3] * sb0 + tb.y * sb1;
+      }
+      la = la * sa0 + mla.y * sa1;
+      lb = lb * sb0 + mlb.y * sb1;
+      ma = na;
+      mb = nb;
+    }
+  }
+
+  // partial (unnormalised o, m, l) of this CTA in its own shared memory
+  if (active && kgrp == 0) {
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
       const int d = nt * 8 + 2 * c4;

@@ -53,10 +53,7 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
   const EpiSmem S = carve_epi<TT>(scratch);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long U = (long)a.w_tiles * a.tok_tiles * a.kc;
-  const long G = gridDim.x;
-  const long c = blockIdx.x;
-  const long u0 = range_start(c, U, G), u1 = range_start(c + 1, U, G);
+  int* live = reinterpret_cast<int*>(misc + 4);  // [0] token tiles processed, [1] token rows of one tile's MMA
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
@@ -65,6 +62,22 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
     mbar_init(fx, 1);
     *abort_flag = 0;
     *fx_armed = 0;
+    // Token tiles past the pass's row count hold no output row.  A
+    // multi-tile launch whose row count was written two or more launches back
+    // (the previous kernel itself waited for that writer before letting this
+    // grid start) reads it now and neither loads nor multiplies those tiles;
+    // when one tile is left it covers only the rows present (B = 2 n_tok
+    // rows).  A single-tile launch takes n_tok from the host's row capacity
+    // and starts without this read.
+    int tiles = a.tok_tiles;
+    int ntok = (a.tok_tiles == 1 && a.n_tok > 0 && a.n_tok < TT && a.n_tok % 8 == 0) ? a.n_tok : TT;
+    if (a.m_early && a.tok_tiles > 1) {
+      const int m = min(max(__ldcg(a.m_dev), 1), a.m_cap);
+      tiles = min(a.tok_tiles, (m + TT - 1) / TT);
+      ntok = tiles == 1 ? min(TT, (m + 7) / 8 * 8) : TT;
+    }
+    live[0] = tiles;
+    live[1] = ntok;
     fence_barrier_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
@@ -72,11 +85,20 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  const int tok_tiles = live[0];
+  const long U = (long)a.w_tiles * tok_tiles * a.kc;
+  const long G = gridDim.x;
+  const long c = blockIdx.x;
+  const long u0 = range_start(c, U, G), u1 = range_start(c + 1, U, G);
   uint32_t armed[C::kStages];  // producer: times each ring slot was armed
   for (int s = 0; s < C::kStages; ++s) armed[s] = 0;
   // ring slots this launch uses, and how many are filled before the PDL wait
   const int R = (a.stages > 0 && a.stages < C::kStages) ? a.stages : C::kStages;
   const int P = (a.pre_stages > 0 && a.pre_stages < R) ? a.pre_stages : R;
+  // token rows a tile's MMA covers: hi/lo pairs are the B rows, so N = 2 n_tok
+  const int n_tok = live[1];
+  const uint32_t b_bytes = (uint32_t)n_tok * 2 * 128;
+  const uint32_t stage_bytes = (uint32_t)C::kABytes + b_bytes;
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -90,7 +112,7 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
       // wake-up with no divisions on the path between the 'empty' signal and
       // the copies.
       int kk = (int)(u0 % a.kc);
-      int w_tile = (int)((u0 / a.kc) / a.tok_tiles), tok_tile = (int)((u0 / a.kc) % a.tok_tiles);
+      int w_tile = (int)((u0 / a.kc) / tok_tiles), tok_tile = (int)((u0 / a.kc) % tok_tiles);
       const __nv_bfloat16* wsrc0 = nullptr;  // packed block base of the current weight tile (A)
       const __nv_bfloat16* wsrc1 = nullptr;  // second half (gate/up pairs)
       const CUtensorMap* wmap0 = nullptr;
@@ -132,19 +154,19 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
         }
       };
       auto issue_b = [&](int s, int kk_, int tok_) {
-        bulk_load(sB + s * C::kBBytes, a.x + (size_t)kk_ * x_blk + (size_t)tok_ * x_tile_off, C::kBBytes, &full[s]);
+        bulk_load(sB + s * C::kBBytes, a.x + (size_t)kk_ * x_blk + (size_t)tok_ * x_tile_off, b_bytes, &full[s]);
       };
       auto advance = [&]() {
         if (++kk == a.kc) {
           kk = 0;
-          if (++tok_tile == a.tok_tiles) { tok_tile = 0; ++w_tile; }
+          if (++tok_tile == tok_tiles) { tok_tile = 0; ++w_tile; }
           set_tile();
         }
       };
       // weights first: they do not depend on the previous kernel
       int pre_kk[C::kStages], pre_tok[C::kStages];
       for (int i = 0; i < npre; ++i) {
-        mbar_arrive_expect_tx(&full[i], C::kStageBytes);
+        mbar_arrive_expect_tx(&full[i], stage_bytes);
         ++armed[i];
         issue_a(i);
         pre_kk[i] = kk;
@@ -161,7 +183,7 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
           *abort_flag = 1;
           break;
         }
-        mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+        mbar_arrive_expect_tx(&full[s], stage_bytes);
         ++armed[s];
         issue_a(s);
         issue_b(s, kk, tok_tile);
@@ -173,7 +195,7 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(kTileN, 2 * TT);
+      const uint32_t idesc = idesc_bf16(kTileN, 2 * n_tok);
       int s = 0;          // ring slot of the next unit
       uint32_t fph = 0;   // its 'full' phase parity
       int seg_i = 0;
@@ -224,7 +246,7 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
       const long ub = u, ue = (t + 1) * a.kc < u1 ? (t + 1) * a.kc : u1;
       u = ue;
       const int ab = seg_i % C::kNumAcc;
-      const int w_tile = (int)(t / a.tok_tiles), tok_tile = (int)(t % a.tok_tiles);
+      const int w_tile = (int)(t / tok_tiles), tok_tile = (int)(t % tok_tiles);
       const int tok_base = tok_tile * TT;
       if (a.ssq_in && tok_base != rs_tok) {
         epi_row_scale<TT>(a, tok_base, et, M, S);
@@ -278,6 +300,7 @@ int gemm_smem_bytes(int tt) {
   switch (tt) {
     case 16: return GemmCfg<16>::kSmem;
     case 64: return GemmCfg<64>::kSmem;
+    case 128: return GemmCfg<128>::kSmem;
     default: return -1;
   }
 }
@@ -308,7 +331,8 @@ void launch_gemm(const GemmArgs& a, int tt, int grid, cudaStream_t s, bool pdl) 
   cudaError_t e;
   switch (tt) {
     case 16: e = launch_tt<16>(a, grid, s, pdl); break;
-    default: e = launch_tt<64>(a, grid, s, pdl); break;
+    case 64: e = launch_tt<64>(a, grid, s, pdl); break;
+    default: e = launch_tt<128>(a, grid, s, pdl); break;
   }
   if (e != cudaSuccess) throw e;
 }

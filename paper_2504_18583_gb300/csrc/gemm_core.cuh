@@ -19,12 +19,14 @@ struct GemmCfg {
   // room on its SM for one CTA of the next launch, which then starts, fills
   // its ring and reaches its PDL wait while this one finishes.  Wider tiles
   // run one CTA per SM and take a deeper ring (~200 KB) instead: with 4 and
-  // 3 stages they kept too few weight bytes in flight per SM.
-  static constexpr int kStages = TT <= 16 ? 5 : (TT <= 32 ? 8 : 6);
+  // 3 stages they kept too few weight bytes in flight per SM.  The 128-token
+  // tile (65-128 rows: one pass over the weights for all of them) fits 4
+  // stages of 48 KB.
+  static constexpr int kStages = TT <= 16 ? 5 : (TT <= 32 ? 8 : (TT <= 64 ? 6 : 4));
   static constexpr int kAccCols = 2 * TT;
-  static constexpr int kNumAcc = (2 * kAccCols <= 256) ? 2 : 1;
+  static constexpr int kNumAcc = (2 * kAccCols <= 512) ? 2 : 1;
   static constexpr int kTmemCols = kNumAcc * kAccCols <= 32 ? 32 : kNumAcc * kAccCols <= 64 ? 64
-                                   : kNumAcc * kAccCols <= 128 ? 128 : 256;
+                                   : kNumAcc * kAccCols <= 128 ? 128 : kNumAcc * kAccCols <= 256 ? 256 : 512;
   static constexpr int kChunks = TT / kEpiTok;
   // scratch after the stage ring
   static constexpr int kBarBytes = 8 * (2 * kStages + 6);  // full, empty, accf x2, acce x2, drain, fix-up

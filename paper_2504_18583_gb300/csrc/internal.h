@@ -42,6 +42,10 @@ struct GemmArgs {
   int seg_rows[kMaxSeg];      // rows of each segment
   int pair;
   int w_tiles, tok_tiles, kc;
+  int n_tok;                  // token rows a tile's MMA covers (multiple of 8, <= the tile; 0: the whole tile):
+                              // a single-tile pass of fewer rows loads and multiplies only those
+  int m_early;                // m_dev was written two or more launches back: read it before the PDL wait and
+                              // skip the token tiles past it (0: process every tile)
   int mode;
   int m_cap;                  // row capacity of the activation/output buffers
   const int* m_dev;           // runtime row count
@@ -97,6 +101,7 @@ struct AttnArgs {
   int hq, hkv, hd, page_size, n_pages;
   int row_blocks;             // row blocks per sequence (grid.y / ...)
   int n_split;                // key splits
+  int nbuf;                   // K/V chunk buffers a CTA keeps (4, or 2 when many units share the SMs)
   float scale;
   __nv_bfloat16* x_out;       // packed [2*rows][hq*hd] hi/lo
   int x_rows;
@@ -108,6 +113,7 @@ struct AttnArgs {
 // of the key splits, and bit kAttnPathSplit0 + n for clusters of n CTAs.
 constexpr uint32_t kAttnPathPush = 1u << 0;
 constexpr uint32_t kAttnPathPull = 1u << 1;
+constexpr uint32_t kAttnPathRing2 = 1u << 2;  // the two-buffer K/V ring variant ran
 constexpr int kAttnPathSplit0 = 3;
 
 

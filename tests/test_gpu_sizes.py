@@ -12,7 +12,7 @@ from _parity import LOGIT_TOL, Pair, greedy_step, sampling_step
 
 pytestmark = pytest.mark.gpu
 
-PUSH, PULL, SPLIT0 = 1 << 0, 1 << 1, 3
+PUSH, PULL, RING2, SPLIT0 = 1 << 0, 1 << 1, 1 << 2, 3
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -43,7 +43,7 @@ def test_long_contexts_pull_combine_and_8_cta_clusters():
         greedy_step(P, step)
     bits = P.eng.attention_paths()
     print("16-CTA clusters: paths", hex(bits), "cluster sizes", split_sizes(bits), "stats", P.stats)
-    assert bits & PULL and not bits & PUSH
+    assert bits & PULL and not bits & PUSH and not bits & RING2
     assert split_sizes(bits) == [16]
     P.eng.set_attention_split_cap(8)
     for step in range(4, 7):
@@ -57,8 +57,11 @@ def test_long_contexts_pull_combine_and_8_cta_clusters():
 def test_batch16_ragged_c3_prompts_two_layers():
     """The batch-16 configuration at its own sizes (16 prompts of 128..2048
     tokens drawn from its seed, K = 6), two layers per model at full width:
-    112 verify and up to 192 draft rows over contexts that differ by 16x;
-    clusters of short sequences push, long ones pull.  Three greedy steps."""
+    112 verify and up to 192 draft rows over contexts that differ by 16x.
+    The key splits are sized by the contexts' total (five splits here, more
+    units than two per SM), so the attention takes its two-buffer K/V ring
+    with four CTAs per SM, and the long sequences' warp pairs split every
+    chunk's keys; the clusters combine by the pull.  Three greedy steps."""
     wl = S.WORKLOADS["8b_batch16"].replace(target=S.TARGET_8B.replace(n_layers=2),
                                            draft=S.DRAFT_1B.replace(n_layers=2), n_new=20)
     print("prompt lengths", wl.prompt_lens())
@@ -69,7 +72,8 @@ def test_batch16_ragged_c3_prompts_two_layers():
         greedy_step(P, step)
     bits = P.eng.attention_paths()
     print("paths", hex(bits), "cluster sizes", split_sizes(bits), "stats", P.stats)
-    assert bits & PULL and bits & PUSH
+    assert bits & PULL and bits & RING2
+    assert split_sizes(bits) == [5]
     assert P.eng.last_status() == 0
 
 
