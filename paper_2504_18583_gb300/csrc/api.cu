@@ -143,8 +143,7 @@ WsOffsets layout_ws(const Dims& D, const pard_limits& lim) {
   o.ssq = L.take((size_t)(D.dmax / 128) * D.MC * 4);
   o.ssqg = L.take((size_t)(D.dmax / 128) * D.MC * 4);
   o.q = L.take((size_t)D.MC * D.qdmax * 4);
-  o.gpart = L.take((size_t)D.sm * 2 * kTileN * (D.MC > 64 ? 128 : 64) * 4);  // two partial tiles per CTA
-  o.gcnt = L.take((size_t)65536 * 4);
+  o.gcnt = L.take((size_t)kMaxGemmTiles * 8);  // one 64-bit arrival mask per output tile
   o.stats_t = L.take((size_t)D.w_tiles * D.MC * 16);
   o.stats_it = L.take((size_t)D.w_tiles * D.MC * 8);
   o.stats_d = L.take((size_t)D.w_tiles * D.MC * 16);
@@ -181,6 +180,7 @@ WsOffsets layout_ws(const Dims& D, const pard_limits& lim) {
   for (int mi = 0; mi < 2; ++mi) o.rope[mi] = L.take((size_t)D.pt_ld * lim.page_size * (D.hdmax / 2) * 8);
   o.g_plen = L.take((size_t)B * 4);
   o.mask_ids = L.take((size_t)std::max(K, 1) * 4);
+  o.gpart = L.take((size_t)D.sm * 2 * kTileN * (D.MC > 64 ? 128 : 64) * 4);  // two partial tiles per CTA
   o.pack_tmp = L.take(kPackTmpBytes);
   o.total = L.total + 256;
   return o;
@@ -321,8 +321,12 @@ GemmArgs gemm_base(pard_ctx* c, int rows_cap, int tt) {
 void run_gemm(pard_ctx* c, GemmArgs& a, int tt, cudaStream_t s) {
   const long U = (long)a.w_tiles * a.tok_tiles * a.kc;
   // at least 8 units (128 KB of weights) a CTA: with fewer, the split-K
-  // finish of a tile gathers partials from too many CTAs
-  const int grid = (int)std::min<long>(c->sm, std::max<long>(1, U / 8));
+  // finish of a tile gathers partials from too many CTAs; and at least
+  // kc / 62 units, so that no tile has more than 63 contributors (the
+  // finisher tracks their arrivals in one 64-bit mask)
+  const long min_units = std::max<long>(8, (a.kc + 61) / 62);
+  const int grid = (int)std::min<long>(c->sm, std::max<long>(1, U / min_units));
+  if ((long)a.w_tiles * a.tok_tiles > kMaxGemmTiles) throw cudaErrorInvalidValue;
   launch_gemm(a, tt, grid, s, true);
   c->launches++;
 }
@@ -659,7 +663,7 @@ pard_status pard_load_weights(pard_ctx** out, const pard_model_cfg* tcfg, const 
     c->mask_ids = c->at<int>(o.mask_ids);
 
     // counters start at zero; the reduction kernels leave them at zero
-    CK(cudaMemsetAsync(c->gcnt, 0, 65536 * 4, s));
+    CK(cudaMemsetAsync(c->gcnt, 0, (size_t)kMaxGemmTiles * 8, s));
     CK(cudaMemsetAsync(c->st.samp_cnt, 0, lim->max_batch * 4, s));
     CK(cudaMemsetAsync(c->status, 0, 4, s));
     CK(cudaMemsetAsync(c->paths, 0, 4, s));

@@ -403,12 +403,15 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
     }
   }
   bar();
-  // Warp roles.  Query vectors are tiled 16 to a warp.  When they fit in two
-  // warps and the unit walks at least kKeyHalvesMinChunks chunks, the other
-  // two warps would idle: instead warps 0-1 take keys 0-15 and warps 2-3
-  // keys 16-31 of every chunk, each pair with its own online-softmax state,
-  // and the pairs' states are merged once after the last chunk.
-  const int ng = ((nqv + 15) / 16 <= 2 && n >= kKeyHalvesMinChunks) ? 2 : 1;
+  // Warp roles.  Query vectors are tiled 16 to a warp.  In the two-buffer
+  // form (passes with many units), when they fit in two warps and the unit
+  // walks at least kKeyHalvesMinChunks chunks, the other two warps would
+  // idle: instead warps 0-1 take keys 0-15 and warps 2-3 keys 16-31 of every
+  // chunk, each pair with its own online-softmax state, and the pairs'
+  // states are merged once after the last chunk.  (The four-buffer form of
+  // batch-1 passes walks one or two chunks a unit and keeps one warp set.)
+  constexpr bool kHalves = NBUF == 2;
+  const int ng = (kHalves && (nqv + 15) / 16 <= 2 && n >= kKeyHalvesMinChunks) ? 2 : 1;
   const int qtile = ng == 2 ? (warp & 1) : warp;
   const int kgrp = ng == 2 ? (warp >> 1) : 0;
   const int qa = qtile * 16 + g, qb = qa + 8;
@@ -444,17 +447,21 @@ __device__ AttnRows attn_unit(const AttnArgs& a, int b, int kvh, int rb, int sp,
       ++issued;
     }
     if (active) {
-      if (ng == 2)
-        attn_chunk<HD, NJ / 2, C::kRowBytes>(sK, sV, kgrp * (kKeyChunk / 2), ch, q_base, posa, posb, a.scale, o, ma,
-                                             mb, la, lb, lane);
-      else
+      if constexpr (kHalves) {
+        if (ng == 2)
+          attn_chunk<HD, NJ / 2, C::kRowBytes>(sK, sV, kgrp * (kKeyChunk / 2), ch, q_base, posa, posb, a.scale, o,
+                                               ma, mb, la, lb, lane);
+        else
+          attn_chunk<HD, NJ, C::kRowBytes>(sK, sV, 0, ch, q_base, posa, posb, a.scale, o, ma, mb, la, lb, lane);
+      } else {
         attn_chunk<HD, NJ, C::kRowBytes>(sK, sV, 0, ch, q_base, posa, posb, a.scale, o, ma, mb, la, lb, lane);
+      }
     }
   }
   bar();  // K/V and Q buffers are reused for the partial results below
 
   float* part = reinterpret_cast<float*>(smem);
-  if (ng == 2) {
+  if (kHalves && ng == 2) {
     // Warps 2-3 hand their state to their twins in warps 0-1 (same lane, same
     // query vectors) through partial rows 32-63, which no push into this
     // CTA's receive area reaches: a unit walking kKeyHalvesMinChunks chunks

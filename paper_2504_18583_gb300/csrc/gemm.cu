@@ -54,6 +54,12 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   int* live = reinterpret_cast<int*>(misc + 4);  // [0] token tiles processed, [1] token rows of one tile's MMA
+  // this CTA's units (recomputed below in the rare launch that drops token tiles)
+  const bool early = a.m_early && a.tok_tiles > 1;
+  const long G = gridDim.x;
+  const long c = blockIdx.x;
+  long U = (long)a.w_tiles * a.tok_tiles * a.kc;
+  long u0 = range_start(c, U, G), u1 = range_start(c + 1, U, G);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
@@ -69,15 +75,12 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
     // when one tile is left it covers only the rows present (B = 2 n_tok
     // rows).  A single-tile launch takes n_tok from the host's row capacity
     // and starts without this read.
-    int tiles = a.tok_tiles;
-    int ntok = (a.tok_tiles == 1 && a.n_tok > 0 && a.n_tok < TT && a.n_tok % 8 == 0) ? a.n_tok : TT;
-    if (a.m_early && a.tok_tiles > 1) {
+    if (early) {
       const int m = min(max(__ldcg(a.m_dev), 1), a.m_cap);
-      tiles = min(a.tok_tiles, (m + TT - 1) / TT);
-      ntok = tiles == 1 ? min(TT, (m + 7) / 8 * 8) : TT;
+      const int tiles = min(a.tok_tiles, (m + TT - 1) / TT);
+      live[0] = tiles;
+      live[1] = tiles == 1 ? min(TT, (m + 7) / 8 * 8) : TT;
     }
-    live[0] = tiles;
-    live[1] = ntok;
     fence_barrier_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
@@ -85,18 +88,20 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const int tok_tiles = live[0];
-  const long U = (long)a.w_tiles * tok_tiles * a.kc;
-  const long G = gridDim.x;
-  const long c = blockIdx.x;
-  const long u0 = range_start(c, U, G), u1 = range_start(c + 1, U, G);
+  const int tok_tiles = early ? live[0] : a.tok_tiles;
+  if (tok_tiles != a.tok_tiles) {
+    U = (long)a.w_tiles * tok_tiles * a.kc;
+    u0 = range_start(c, U, G);
+    u1 = range_start(c + 1, U, G);
+  }
   uint32_t armed[C::kStages];  // producer: times each ring slot was armed
   for (int s = 0; s < C::kStages; ++s) armed[s] = 0;
   // ring slots this launch uses, and how many are filled before the PDL wait
   const int R = (a.stages > 0 && a.stages < C::kStages) ? a.stages : C::kStages;
   const int P = (a.pre_stages > 0 && a.pre_stages < R) ? a.pre_stages : R;
   // token rows a tile's MMA covers: hi/lo pairs are the B rows, so N = 2 n_tok
-  const int n_tok = live[1];
+  const int n_tok = early ? live[1]
+                           : ((a.tok_tiles == 1 && a.n_tok > 0 && a.n_tok < TT && a.n_tok % 8 == 0) ? a.n_tok : TT);
   const uint32_t b_bytes = (uint32_t)n_tok * 2 * 128;
   const uint32_t stage_bytes = (uint32_t)C::kABytes + b_bytes;
 
@@ -286,7 +291,8 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
       umma_commit(drain);
       mbar_drain(drain, 0);
     }
-    if (threadIdx.x == 64 && *fx_armed) mbar_drain(fx, 0);
+    // fx_armed: 1 + the staging round whose copies may be in flight
+    if (threadIdx.x == 64 && *fx_armed) mbar_drain(fx, (uint32_t)((*fx_armed - 1) & 1));
     __syncthreads();
   }
   if (warp == 1) {

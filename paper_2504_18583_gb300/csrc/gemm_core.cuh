@@ -408,16 +408,22 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
 }
 
 
-// Bounded wait until *p >= target, with acquire semantics on success.
-__device__ __forceinline__ bool wait_count(const int* p, int target, volatile int* abort) {
-  if (ld_acquire_s32(p) >= target) return true;
+// Bounded wait until every bit of `all` is set in *p, with acquire semantics
+// on success.
+__device__ __forceinline__ bool wait_mask(const unsigned long long* p, unsigned long long all, volatile int* abort) {
+  if ((ld_acquire_u64(p) & all) == all) return true;
   const unsigned long long t0 = globaltimer();
   while (true) {
-    if (ld_acquire_s32(p) >= target) return true;
+    if ((ld_acquire_u64(p) & all) == all) return true;
     if (*abort) return false;
     if (globaltimer() - t0 > kWaitLimitNs) return false;
   }
 }
+// bits of contributors 1..n of a tile (bit k - 1: the k-th after the finisher)
+__device__ __forceinline__ unsigned long long contrib_bits(int n) { return n >= 64 ? ~0ull : ((1ull << n) - 1); }
+// 4-token groups of a 16-token chunk that hold some of the pass's M rows: a
+// partial tile stores and copies only those ([chunk][j4][row] layout)
+__device__ __forceinline__ int chunk_groups(int M, int tok0) { return min(4, max(0, (M - tok0 + 3) / 4)); }
 
 // Split-K with a designated finisher (per-phase kernel).  The first CTA of a
 // tile in CTA order, cf, finishes it.  Its share of the tile is the last
@@ -425,12 +431,19 @@ __device__ __forceinline__ bool wait_count(const int* p, int target, volatile in
 // end), so when its epilogue gets there every MMA of the CTA has completed and
 // the stage ring is idle.  The other contributors store their partial, make
 // one release increment of the tile's counter and move on without a round
-// trip.  cf waits for the cl - cf increments, pulls every partial into the
-// ring with one bulk copy each (a single round trip for the whole tile) and
-// sums in CTA order, itself first (deterministic).  pre0: epi_pre of the segment's first
-// chunk, taken by the caller before the accumulator was ready; only read for
-// a whole tile or by cf.  ring/ring_bytes: the stage ring; fx: an mbarrier
-// used once per launch; fx_armed: set while its copies are in flight.
+// trip.  Contributor k (the k-th CTA after cf) stores its partial and sets
+// bit k - 1 of the tile's arrival mask with one release OR; cf copies each
+// partial into the ring as soon as its bit is seen (so the copies of early
+// contributors overlap the wait for late ones) and sums in CTA order,
+// itself first (deterministic).  With many chunks (wide tiles) the copies
+// go in rounds of chunks once every bit is set.  pre0: epi_pre of the segment's first chunk, taken by the
+// caller before the accumulator was ready; only read for a whole tile or by
+// cf.  ring/ring_bytes: the stage ring; fx: an mbarrier whose phase r is
+// round r of the one split tile a CTA finishes; fx_armed: 1 + the round
+// whose copies may be in flight (0: none).  Partials hold only the 4-token
+// groups with output rows (chunk_groups).  The arrival masks live in
+// a.counters (64-bit words, tile t at word t; the host keeps every tile's
+// contributors at 64 or fewer) and are cleared by the finisher.
 template <int TT>
 __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, long u0, long U, long G, long c,
                                   uint32_t tbase, int w_tile, int tok_base, int fr, int et, int M, const EpiSmem& S,
@@ -457,6 +470,7 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
     return true;
   }
   const long cf = owner_of(t * a.kc, U, G), cl = owner_of((t + 1) * a.kc - 1, U, G);
+  unsigned long long* mask = reinterpret_cast<unsigned long long*>(a.counters) + t;
   if (c != cf) {
     const int slot = (ub == u0) ? 0 : 1;
     float* mine = a.partials + ((size_t)c * 2 + slot) * kTileF;
@@ -464,86 +478,191 @@ __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, l
     for (int ch = 0; ch < nch; ++ch) {
       uint32_t r[32];
       tmem_ld32(tbase + ch * 32, r);
+      const int ng = chunk_groups(M, tok_base + ch * kEpiTok);
       // [chunk][j4][row] float4s: a warp's accesses are 512 contiguous bytes
       float4* dst = reinterpret_cast<float4*>(mine + (size_t)ch * kTileN * kEpiTok) + fr;
 #pragma unroll
       for (int j4 = 0; j4 < 4; ++j4)
-        dst[j4 * kTileN] = make_float4(__uint_as_float(r[8 * j4 + 0]) + __uint_as_float(r[8 * j4 + 1]),
-                              __uint_as_float(r[8 * j4 + 2]) + __uint_as_float(r[8 * j4 + 3]),
-                              __uint_as_float(r[8 * j4 + 4]) + __uint_as_float(r[8 * j4 + 5]),
-                              __uint_as_float(r[8 * j4 + 6]) + __uint_as_float(r[8 * j4 + 7]));
+        if (j4 < ng)
+          dst[j4 * kTileN] = make_float4(__uint_as_float(r[8 * j4 + 0]) + __uint_as_float(r[8 * j4 + 1]),
+                                __uint_as_float(r[8 * j4 + 2]) + __uint_as_float(r[8 * j4 + 3]),
+                                __uint_as_float(r[8 * j4 + 4]) + __uint_as_float(r[8 * j4 + 5]),
+                                __uint_as_float(r[8 * j4 + 6]) + __uint_as_float(r[8 * j4 + 7]));
     }
-    // the barrier orders every thread's partial before the one release
-    // increment (cumulative)
+    // the barrier orders every thread's partial before the one release OR
+    // (cumulative)
     epi_bar();
-    if (et == 0) red_release_add(reinterpret_cast<unsigned*>(&a.counters[t]), 1u);
+    if (et == 0) red_release_or64(mask, 1ull << (c - cf - 1));
     return true;
   }
-  const int n_other = (int)(cl - cf);
-  const uint32_t part_bytes = (uint32_t)nch * kChF * 4;  // of one contributor: its first nch chunks
-  const bool staged = (uint32_t)n_other * part_bytes <= ring_bytes;
-  if (et == 0) {
-    const bool ok = wait_count(&a.counters[t], n_other, abort_flag);
-    if (!ok) set_status(a.status, ST_TIMEOUT_EPI);
-    if (ok && staged && nch > 0) {
-      // the partials were written through the generic proxy; the copies read
-      // them through the async proxy
-      fence_proxy_async();
-      *fx_armed = 1;
-      mbar_arrive_expect_tx(fx, (uint32_t)n_other * part_bytes);
-      for (int k = 0; k < n_other; ++k) {
-        const long cc = cf + 1 + k;
-        const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
-        bulk_load(ring + (size_t)k * nch * kChF, a.partials + ((size_t)cc * 2 + sl) * kTileF, part_bytes, fx);
-      }
-    }
-    bcast[0] = ok ? 1 : 0;
-  }
-  epi_bar();
-  if (!bcast[0]) {
-    *abort_flag = 1;
-    return false;
-  }
-  const bool late = staged && nch > 0 && !mbar_wait(fx, 0, abort_flag);
-  if (epi_bar_any(late)) {
-    if (et == 0) set_status(a.status, ST_TIMEOUT_EPI);
-    *abort_flag = 1;
-    return false;
-  }
-  EpiPre pre = pre0;
-#pragma unroll 1
-  for (int ch = 0; ch < nch; ++ch) {
-    if (ch > 0) pre = epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M);
-    uint32_t r[32];
-    tmem_ld32(tbase + ch * 32, r);
-    float v[kEpiTok];
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
-    const size_t off = (size_t)ch * kTileN * kEpiTok;
-    for (int k = 0; k < n_other; ++k) {
-      float4 pv[4];
+  if constexpr (C::kChunks == 1) {
+    // 16-token tile: one chunk, so one staging round (the partials of up to
+    // ring_bytes / 8 KB contributors) or direct loads
+    const int n_other = (int)(cl - cf);
+    // bytes copied of one contributor: the 4-token groups of its chunk with output rows
+    const uint32_t part_bytes = nch > 0 ? (uint32_t)chunk_groups(M, tok_base) * kTileN * 16 : 0u;
+    const bool staged = nch > 0 && (uint32_t)n_other * kChF * 4 <= ring_bytes;
+    if (et == 0) {
+      const unsigned long long all = contrib_bits(n_other);
+      bool ok = true;
       if (staged) {
-        const float4* p = reinterpret_cast<const float4*>(ring + (size_t)k * nch * kChF + off) + fr;
-#pragma unroll
-        for (int j4 = 0; j4 < 4; ++j4) pv[j4] = p[j4 * kTileN];
+        *fx_armed = 1;
+        mbar_arrive_expect_tx(fx, (uint32_t)n_other * part_bytes);
+        // copy each contributor's partial as soon as its bit is seen
+        unsigned long long seen = 0;
+        const unsigned long long t0 = globaltimer();
+        while (seen != all) {
+          const unsigned long long m = ld_acquire_u64(mask) & all;
+          unsigned long long nw = m & ~seen;
+          if (nw) {
+            // the partials were written through the generic proxy; the copies
+            // read them through the async proxy
+            fence_proxy_async();
+            while (nw) {
+              const int k = __ffsll((long long)nw) - 1;
+              nw &= nw - 1;
+              const long cc = cf + 1 + k;
+              const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
+              bulk_load(ring + (size_t)k * kChF, a.partials + ((size_t)cc * 2 + sl) * kTileF, part_bytes, fx);
+            }
+            seen = m;
+          } else if (*abort_flag || globaltimer() - t0 > kWaitLimitNs) {
+            ok = false;
+            break;
+          }
+        }
       } else {
-        const long cc = cf + 1 + k;
-        const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
-        const float4* p = reinterpret_cast<const float4*>(a.partials + ((size_t)cc * 2 + sl) * kTileF + off) + fr;
-#pragma unroll
-        for (int j4 = 0; j4 < 4; ++j4) pv[j4] = __ldcg(p + j4 * kTileN);
+        ok = wait_mask(mask, all, abort_flag);
       }
-#pragma unroll
-      for (int j4 = 0; j4 < 4; ++j4) {
-        v[4 * j4 + 0] += pv[j4].x;
-        v[4 * j4 + 1] += pv[j4].y;
-        v[4 * j4 + 2] += pv[j4].z;
-        v[4 * j4 + 3] += pv[j4].w;
-      }
+      if (!ok) set_status(a.status, ST_TIMEOUT_EPI);
+      bcast[0] = ok ? 1 : 0;
     }
-    epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S, pre);
+    epi_bar();
+    if (!bcast[0]) {
+      *abort_flag = 1;
+      return false;
+    }
+    const bool late = staged && nch > 0 && !mbar_wait(fx, 0, abort_flag);
+    if (epi_bar_any(late)) {
+      if (et == 0) set_status(a.status, ST_TIMEOUT_EPI);
+      *abort_flag = 1;
+      return false;
+    }
+    EpiPre pre = pre0;
+  #pragma unroll 1
+    for (int ch = 0; ch < nch; ++ch) {
+      if (ch > 0) pre = epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M);
+      uint32_t r[32];
+      tmem_ld32(tbase + ch * 32, r);
+      float v[kEpiTok];
+  #pragma unroll
+      for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
+      const size_t off = (size_t)ch * kTileN * kEpiTok;
+      for (int k = 0; k < n_other; ++k) {
+        float4 pv[4];
+        if (staged) {
+          const float4* p = reinterpret_cast<const float4*>(ring + (size_t)k * kChF + off) + fr;
+  #pragma unroll
+          for (int j4 = 0; j4 < 4; ++j4) pv[j4] = p[j4 * kTileN];
+        } else {
+          const long cc = cf + 1 + k;
+          const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
+          const float4* p = reinterpret_cast<const float4*>(a.partials + ((size_t)cc * 2 + sl) * kTileF + off) + fr;
+  #pragma unroll
+          for (int j4 = 0; j4 < 4; ++j4) pv[j4] = __ldcg(p + j4 * kTileN);
+        }
+  #pragma unroll
+        for (int j4 = 0; j4 < 4; ++j4) {
+          v[4 * j4 + 0] += pv[j4].x;
+          v[4 * j4 + 1] += pv[j4].y;
+          v[4 * j4 + 2] += pv[j4].z;
+          v[4 * j4 + 3] += pv[j4].w;
+        }
+      }
+      epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S, pre);
+    }
+  } else {
+    const int n_other = (int)(cl - cf);
+    // Partials are staged in the idle ring in rounds of chunks: each round one
+    // bulk copy per contributor brings the same run of chunks of every
+    // partial ([chunk][j4][row] layout: a run of chunks is contiguous), so a
+    // tile with many contributors or many chunks costs a few round trips
+    // instead of one L2 load chain per chunk.
+    const uint32_t ch_bytes = (uint32_t)kChF * 4;
+    int per_round = n_other > 0 ? (int)(ring_bytes / ((uint32_t)n_other * ch_bytes)) : nch;
+    if (per_round > nch) per_round = nch;
+    const bool staged = per_round > 0 && nch > 0;
+    if (et == 0) {
+      const bool ok = wait_mask(mask, contrib_bits(n_other), abort_flag);
+      if (!ok) set_status(a.status, ST_TIMEOUT_EPI);
+      bcast[0] = ok ? 1 : 0;
+    }
+    epi_bar();
+    if (!bcast[0]) {
+      *abort_flag = 1;
+      return false;
+    }
+    EpiPre pre = pre0;
+    const int step = staged ? per_round : nch;
+    for (int r0 = 0, round = 0; r0 < nch; r0 += step, ++round) {
+      const int r1 = min(nch, r0 + step), nr = r1 - r0;
+      if (staged) {
+        if (et == 0) {
+          // the partials were written through the generic proxy (and the ring
+          // read through it by the previous round); the copies use the async proxy
+          fence_proxy_async();
+          *fx_armed = round + 1;
+          mbar_arrive_expect_tx(fx, (uint32_t)n_other * nr * ch_bytes);
+          for (int k = 0; k < n_other; ++k) {
+            const long cc = cf + 1 + k;
+            const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
+            bulk_load(ring + (size_t)k * nr * kChF, a.partials + ((size_t)cc * 2 + sl) * kTileF + (size_t)r0 * kChF,
+                      (uint32_t)nr * ch_bytes, fx);
+          }
+        }
+        const bool late = !mbar_wait(fx, (uint32_t)(round & 1), abort_flag);
+        if (epi_bar_any(late)) {
+          if (et == 0) set_status(a.status, ST_TIMEOUT_EPI);
+          *abort_flag = 1;
+          return false;
+        }
+      }
+  #pragma unroll 1
+      for (int ch = r0; ch < r1; ++ch) {
+        if (ch > 0) pre = epi_pre(a, w_tile, tok_base + ch * kEpiTok, et, M);
+        uint32_t r[32];
+        tmem_ld32(tbase + ch * 32, r);
+        float v[kEpiTok];
+  #pragma unroll
+        for (int j = 0; j < kEpiTok; ++j) v[j] = __uint_as_float(r[2 * j]) + __uint_as_float(r[2 * j + 1]);
+        for (int k = 0; k < n_other; ++k) {
+          float4 pv[4];
+          if (staged) {
+            const float4* p = reinterpret_cast<const float4*>(ring + ((size_t)k * nr + (ch - r0)) * kChF) + fr;
+  #pragma unroll
+            for (int j4 = 0; j4 < 4; ++j4) pv[j4] = p[j4 * kTileN];
+          } else {
+            const long cc = cf + 1 + k;
+            const int sl = range_start(cc, U, G) >= t * a.kc ? 0 : 1;
+            const float4* p = reinterpret_cast<const float4*>(a.partials + ((size_t)cc * 2 + sl) * kTileF +
+                                                              (size_t)ch * kChF) + fr;
+  #pragma unroll
+            for (int j4 = 0; j4 < 4; ++j4) pv[j4] = __ldcg(p + j4 * kTileN);
+          }
+  #pragma unroll
+          for (int j4 = 0; j4 < 4; ++j4) {
+            v[4 * j4 + 0] += pv[j4].x;
+            v[4 * j4 + 1] += pv[j4].y;
+            v[4 * j4 + 2] += pv[j4].z;
+            v[4 * j4 + 3] += pv[j4].w;
+          }
+        }
+        epi_chunk(a, v, w_tile, tok_base + ch * kEpiTok, ch * kEpiTok, fr, et, M, S, pre);
+      }
+      if (staged && r1 < nch) epi_bar();  // the ring is read out before the next round's copies
+    }
   }
-  if (et == 0) a.counters[t] = 0;
+  if (et == 0) *mask = 0ull;
   return true;
 }
 

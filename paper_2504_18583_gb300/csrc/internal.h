@@ -50,7 +50,7 @@ struct GemmArgs {
   int m_cap;                  // row capacity of the activation/output buffers
   const int* m_dev;           // runtime row count
   float* partials;
-  int* counters;
+  int* counters;              // split-K arrival masks: 64-bit word per output tile, zero between launches
   uint32_t* status;
   int stages;                 // ring slots used (0: all the kernel has)
   int pre_stages;             // slots filled before waiting on the previous kernel (0: stages)
@@ -199,6 +199,7 @@ struct AcceptArgs {
   uint32_t* status;        // sticky device status word (null: none)
 };
 
+constexpr int kMaxGemmTiles = 32768;  // output tiles (weight tile x token tile) of one GEMM launch
 constexpr int kMaxQVRows = 64;          // query vectors of one attention work unit
 constexpr int kMaxAttnSplit = 16;       // key splits (CTAs of one cluster) of one attention work unit
 
