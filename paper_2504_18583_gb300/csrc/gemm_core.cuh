@@ -31,7 +31,7 @@ struct GemmCfg {
   // scratch after the stage ring
   static constexpr int kBarBytes = 8 * (2 * kStages + 6);  // full, empty, accf x2, acce x2, drain, fix-up
   static constexpr int kMiscBytes = 64;
-  static constexpr int kScratchFloats = TT + 4 * 64 + 16 + kEpiTok * kTileN + 3 * kEpiTok;
+  static constexpr int kScratchFloats = TT + kEpiTok * kTileN + 3 * kEpiTok;
   static constexpr int kSmem = 1024 + kStages * kStageBytes + kBarBytes + kMiscBytes + 4 * kScratchFloats;
 };
 
@@ -64,12 +64,7 @@ __device__ __forceinline__ int seg_of(const GemmArgs& a, int w_tile) {
 
 struct EpiSmem {
   float* rs;     // [TT]   RMS row scale
-  float* red;    // [4][16]
-  int* redi;     // [4][16]
-  float* red2;   // [4][16]
-  int* redi2;    // [4][16]
-  float* tmx;    // [16]
-  float* xch;    // [16][128]
+  float* xch;    // [16][128] the chunk's accumulator, exchanged to row-major (16-byte aligned)
   int* ri;       // [3][16] per-row facts of the chunk, loaded once by 16 threads
 };
 
@@ -78,12 +73,7 @@ template <int TT>
 __device__ __forceinline__ EpiSmem carve_epi(float* p) {
   EpiSmem S;
   S.rs = p;
-  S.red = S.rs + TT;
-  S.redi = reinterpret_cast<int*>(S.red + 64);
-  S.red2 = reinterpret_cast<float*>(S.redi + 64);
-  S.redi2 = reinterpret_cast<int*>(S.red2 + 64);
-  S.tmx = reinterpret_cast<float*>(S.redi2 + 64);
-  S.xch = S.tmx + 16;
+  S.xch = S.rs + TT;
   S.ri = reinterpret_cast<int*>(S.xch + kEpiTok * kTileN);
   return S;
 }
@@ -176,7 +166,6 @@ static __device__ __forceinline__ EpiPre epi_pre(const GemmArgs& a, int w_tile, 
 // pre holds the chunk's result-independent loads (epi_pre).
 static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_tile, int tok0, int rs_off, int fr,
                           int et, int M, const EpiSmem& S, const EpiPre& pre) {
-  const int q = fr >> 5, lane = fr & 31;
   if (a.ssq_in) {
 #pragma unroll
     for (int j = 0; j < kEpiTok; ++j) v[j] *= S.rs[rs_off + j];
@@ -324,8 +313,6 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
     }
     epi_bar();
   } else {  // MODE_LOGITS
-    const int vi = w_tile * kTileN + fr;
-    const bool valid = vi < a.vocab;
     const float T = a.call->temp;
     const bool sample = a.call->sample != 0 && a.row_gi != nullptr;
     // row facts of the chunk: logits row (-1: none), Gumbel index (-1: none), sequence
@@ -334,76 +321,79 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
       S.ri[kEpiTok + et] = pre.ri[1];
       S.ri[2 * kEpiTok + et] = pre.ri[2];
     }
+#pragma unroll
+    for (int j = 0; j < kEpiTok; ++j) S.xch[j * kTileN + fr] = v[j];
     epi_bar();
-    float x[kEpiTok];
+    // Row-major phase: thread et reduces token jl's 16 vocabulary entries
+    // c16 .. c16 + 15 of the tile in registers, then merges with the other 7
+    // threads of its token (adjacent lanes) by three shuffles.
+    const int m = tok0 + jl;
+    const int n0 = w_tile * kTileN + c16;
+    float x[16];
+    {
+      const float4* xr = reinterpret_cast<const float4*>(S.xch + jl * kTileN + c16);
 #pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      x[j] = valid ? v[j] : -INFINITY;
-      const int orow = S.ri[j];
-      if (a.logits && valid && orow >= 0) a.logits[(size_t)orow * a.vocab + vi] = v[j];
+      for (int i4 = 0; i4 < 4; ++i4) {
+        const float4 q4 = xr[i4];
+        x[4 * i4 + 0] = q4.x; x[4 * i4 + 1] = q4.y; x[4 * i4 + 2] = q4.z; x[4 * i4 + 3] = q4.w;
+      }
     }
-    // tile max and argmax per row
+    const int orow = S.ri[jl];
+    if (a.logits && orow >= 0 && m < M) {
+      float* lp = a.logits + (size_t)orow * a.vocab + n0;
+      if (n0 + 16 <= a.vocab && (a.vocab & 3) == 0) {
 #pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      float mv = x[j];
-      int mi = valid ? vi : INT_MAX;
-      warp_argmax(mv, mi);
-      if (lane == 0) { S.red[q * 16 + j] = mv; S.redi[q * 16 + j] = mi; }
+        for (int i4 = 0; i4 < 4; ++i4)
+          reinterpret_cast<float4*>(lp)[i4] = make_float4(x[4 * i4], x[4 * i4 + 1], x[4 * i4 + 2], x[4 * i4 + 3]);
+      } else {
+        for (int i = 0; i < 16 && n0 + i < a.vocab; ++i) lp[i] = x[i];
+      }
     }
-    // Gumbel-max draw per row (sampling draft rows only)
+    // tile max and argmax (lowest index on ties) of token jl
+    float mv = -INFINITY;
+    int mi = INT_MAX;
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (n0 + i < a.vocab) argmax_merge(mv, mi, x[i], n0 + i);
+#pragma unroll
+    for (int o = 4; o > 0; o >>= 1) {
+      const float v2 = __shfl_xor_sync(0xffffffffu, mv, o);
+      const int i2 = __shfl_xor_sync(0xffffffffu, mi, o);
+      argmax_merge(mv, mi, v2, i2);
+    }
+    // sum of exp((x - max) / T) over the tile
+    float se = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) se += (n0 + i < a.vocab) ? expf(x[i] / T - mv / T) : 0.f;
+    se += __shfl_xor_sync(0xffffffffu, se, 4);
+    se += __shfl_xor_sync(0xffffffffu, se, 2);
+    se += __shfl_xor_sync(0xffffffffu, se, 1);
+    // Gumbel-max draw of the tile (sampling draft rows only)
+    float gv = -INFINITY;
+    int gi = INT_MAX;
     if (sample) {
-#pragma unroll 1
-      for (int j = 0; j < kEpiTok; ++j) {
-        const int m = tok0 + j;
-        float gv = -INFINITY;
-        int gi = INT_MAX;
-        if (m < M && valid) {
-          const int ri = S.ri[kEpiTok + j];
-          if (ri >= 0) {
-            gv = gumbel_score(x[j], T, a.call->seed, (uint32_t)a.gumbel_stream, a.call->step,
-                              (uint32_t)S.ri[2 * kEpiTok + j], (uint32_t)ri, (uint32_t)vi);
-            gi = vi;
-          }
-        }
-        warp_argmax(gv, gi);
-        if (lane == 0) { S.red2[q * 16 + j] = gv; S.redi2[q * 16 + j] = gi; }
+      const int ri = S.ri[kEpiTok + jl];
+      if (m < M && ri >= 0) {
+        const uint32_t sq = (uint32_t)S.ri[2 * kEpiTok + jl];
+        for (int i = 0; i < 16; ++i)
+          if (n0 + i < a.vocab)
+            argmax_merge(gv, gi, gumbel_score(x[i], T, a.call->seed, (uint32_t)a.gumbel_stream, a.call->step, sq,
+                                              (uint32_t)ri, (uint32_t)(n0 + i)),
+                         n0 + i);
       }
-    }
-    epi_bar();
-    if (et < kEpiTok) {
-      float mv = S.red[et];
-      int mi = S.redi[et];
-      for (int qq = 1; qq < 4; ++qq) argmax_merge(mv, mi, S.red[qq * 16 + et], S.redi[qq * 16 + et]);
-      S.tmx[et] = mv;
-      S.redi[et] = mi;  // keep the tile argmax
-      if (sample) {
-        float gv = S.red2[et];
-        int gi = S.redi2[et];
-        for (int qq = 1; qq < 4; ++qq) argmax_merge(gv, gi, S.red2[qq * 16 + et], S.redi2[qq * 16 + et]);
-        S.red2[et] = gv;
-        S.redi2[et] = gi;
-      }
-    }
-    epi_bar();
-    float e[kEpiTok];
 #pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) e[j] = valid ? expf(x[j] / T - S.tmx[j] / T) : 0.f;
-#pragma unroll
-    for (int j = 0; j < kEpiTok; ++j) {
-      const float s = warp_sum(e[j]);
-      if (lane == 0) S.red[q * 16 + j] = s;
-    }
-    epi_bar();
-    if (et < kEpiTok) {
-      const int m = tok0 + et;
-      if (m < M) {
-        const float se = ((S.red[et] + S.red[16 + et]) + S.red[32 + et]) + S.red[48 + et];
-        const size_t o = (size_t)w_tile * a.m_cap + m;
-        a.stats[o] = make_float4(S.tmx[et], se, sample ? S.red2[et] : -INFINITY, 0.f);
-        a.stats_i[o] = make_int2(S.redi[et], sample ? S.redi2[et] : -1);
+      for (int o = 4; o > 0; o >>= 1) {
+        const float v2 = __shfl_xor_sync(0xffffffffu, gv, o);
+        const int i2 = __shfl_xor_sync(0xffffffffu, gi, o);
+        argmax_merge(gv, gi, v2, i2);
       }
     }
-    epi_bar();
+    if ((et & 7) == 0 && m < M) {
+      const size_t o = (size_t)w_tile * a.m_cap + m;
+      a.stats[o] = make_float4(mv, se, sample ? gv : -INFINITY, 0.f);
+      a.stats_i[o] = make_int2(mi, sample ? gi : -1);
+    }
+    epi_bar();  // S.xch and the row facts are rewritten by the next chunk
   }
 }
 
@@ -429,21 +419,21 @@ __device__ __forceinline__ int chunk_groups(int M, int tok0) { return min(4, max
 // tile in CTA order, cf, finishes it.  Its share of the tile is the last
 // segment of its range (the tile starts inside the range and runs past its
 // end), so when its epilogue gets there every MMA of the CTA has completed and
-// the stage ring is idle.  The other contributors store their partial, make
-// one release increment of the tile's counter and move on without a round
-// trip.  Contributor k (the k-th CTA after cf) stores its partial and sets
+// the stage ring is idle.  The other contributors move on without a round
+// trip: contributor k (the k-th CTA after cf) stores its partial and sets
 // bit k - 1 of the tile's arrival mask with one release OR; cf copies each
 // partial into the ring as soon as its bit is seen (so the copies of early
-// contributors overlap the wait for late ones) and sums in CTA order,
-// itself first (deterministic).  With many chunks (wide tiles) the copies
-// go in rounds of chunks once every bit is set.  pre0: epi_pre of the segment's first chunk, taken by the
-// caller before the accumulator was ready; only read for a whole tile or by
-// cf.  ring/ring_bytes: the stage ring; fx: an mbarrier whose phase r is
-// round r of the one split tile a CTA finishes; fx_armed: 1 + the round
-// whose copies may be in flight (0: none).  Partials hold only the 4-token
-// groups with output rows (chunk_groups).  The arrival masks live in
-// a.counters (64-bit words, tile t at word t; the host keeps every tile's
-// contributors at 64 or fewer) and are cleared by the finisher.
+// contributors overlap the wait for late ones), sums the others' partials in
+// CTA order and adds them to its own (deterministic).  With many chunks
+// (wide tiles) the copies go in rounds of chunks once every bit is set.
+// pre0: epi_pre of the segment's first chunk, taken by the caller before the
+// accumulator was ready; only read for a whole tile or by cf.
+// ring/ring_bytes: the stage ring; fx: an mbarrier whose phase r is round r
+// of the one split tile a CTA finishes; fx_armed: 1 + the round whose copies
+// may be in flight (0: none).  Partials hold only the 4-token groups with
+// output rows (chunk_groups).  The arrival masks live in a.counters (64-bit
+// words, tile t at word t; the host keeps every tile's contributors at 64 or
+// fewer) and are cleared by the finisher.
 template <int TT>
 __device__ bool epi_segment_owned(const GemmArgs& a, long t, long ub, long ue, long u0, long U, long G, long c,
                                   uint32_t tbase, int w_tile, int tok_base, int fr, int et, int M, const EpiSmem& S,
