@@ -44,7 +44,12 @@ __global__ void __launch_bounds__(192, TT <= 16 ? 2 : 1) gemm_kernel(const __gri
   uint64_t* acce = accf + 2;
   uint64_t* drain = acce + 2;
   uint64_t* fx = drain + 1;  // split-K finish: partials pulled into the ring
-  uint32_t* misc = reinterpret_cast<uint32_t*>(drain + 2);
+  // the barrier block is rounded to 16 bytes: the epilogue scratch after
+  // misc takes 16-byte vector accesses
+  uint32_t* misc = reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(full) + C::kBarBytes);
+  static_assert(C::kStages * C::kStageBytes % 16 == 0 && C::kBarBytes % 16 == 0 && C::kMiscBytes % 16 == 0 &&
+                    TT % 4 == 0,
+                "epilogue scratch alignment");
   uint32_t* tmem_slot = misc;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
   int* bcast = reinterpret_cast<int*>(misc + 2);

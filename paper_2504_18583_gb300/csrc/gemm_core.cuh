@@ -29,7 +29,8 @@ struct GemmCfg {
                                    : kNumAcc * kAccCols <= 128 ? 128 : kNumAcc * kAccCols <= 256 ? 256 : 512;
   static constexpr int kChunks = TT / kEpiTok;
   // scratch after the stage ring
-  static constexpr int kBarBytes = 8 * (2 * kStages + 6);  // full, empty, accf x2, acce x2, drain, fix-up
+  // full, empty, accf x2, acce x2, drain, fix-up; rounded to 16 bytes
+  static constexpr int kBarBytes = (8 * (2 * kStages + 6) + 15) / 16 * 16;
   static constexpr int kMiscBytes = 64;
   static constexpr int kScratchFloats = TT + kEpiTok * kTileN + 3 * kEpiTok;
   static constexpr int kSmem = 1024 + kStages * kStageBytes + kBarBytes + kMiscBytes + 4 * kScratchFloats;
@@ -423,8 +424,8 @@ __device__ __forceinline__ int chunk_groups(int M, int tok0) { return min(4, max
 // trip: contributor k (the k-th CTA after cf) stores its partial and sets
 // bit k - 1 of the tile's arrival mask with one release OR; cf copies each
 // partial into the ring as soon as its bit is seen (so the copies of early
-// contributors overlap the wait for late ones), sums the others' partials in
-// CTA order and adds them to its own (deterministic).  With many chunks
+// contributors overlap the wait for late ones) and adds them to its own in
+// CTA order (deterministic).  With many chunks
 // (wide tiles) the copies go in rounds of chunks once every bit is set.
 // pre0: epi_pre of the segment's first chunk, taken by the caller before the
 // accumulator was ready; only read for a whole tile or by cf.
