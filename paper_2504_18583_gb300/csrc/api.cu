@@ -349,8 +349,9 @@ AttnGeom attn_geometry(pard_ctx* c, int mi, int rows_per_seq, int batch) {
   if (batch > 1 && (int)c->ctx_est.size() >= batch) {
     // Ragged contexts: the kernel lasts as long as the longest sequence's
     // units, which walk its chunks / n_split each.  Split until that share is
-    // no longer than the average CTA's share of all units' chunks at two
-    // CTAs per SM (more splits only add per-CTA start-up and combine work).
+    // no longer than the average CTA's share of all units' chunks at four
+    // CTAs per SM (the two-buffer form such passes take; more splits only
+    // add per-CTA start-up and combine work).
     long total = 0, longest = 0;
     for (int b = 0; b < batch; ++b) {
       const long ch = (c->ctx_est[b] + 31) / 32;
@@ -358,7 +359,7 @@ AttnGeom attn_geometry(pard_ctx* c, int mi, int rows_per_seq, int batch) {
       longest = std::max(longest, ch);
     }
     total *= (long)cf.n_kv_heads * g.row_blocks;
-    const long bal = total > 0 ? (longest * 2 * c->sm + total - 1) / total : 1;
+    const long bal = total > 0 ? (longest * 4 * c->sm + total - 1) / total : 1;
     g.n_split = std::max<long>(g.n_split, std::min<long>({bal, (long)c->attn_split_cap, (long)n_kt}));
   }
   return g;

@@ -198,10 +198,11 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
         float hn[16];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          hn[4 * i + 0] = hv[i].x + xv[4 * i + 0];
-          hn[4 * i + 1] = hv[i].y + xv[4 * i + 1];
-          hn[4 * i + 2] = hv[i].z + xv[4 * i + 2];
-          hn[4 * i + 3] = hv[i].w + xv[4 * i + 3];
+          const float4 x4 = reinterpret_cast<const float4*>(xv)[i];  // xv: 16-float aligned
+          hn[4 * i + 0] = hv[i].x + x4.x;
+          hn[4 * i + 1] = hv[i].y + x4.y;
+          hn[4 * i + 2] = hv[i].z + x4.z;
+          hn[4 * i + 3] = hv[i].w + x4.w;
           reinterpret_cast<float4*>(hp)[i] = make_float4(hn[4 * i], hn[4 * i + 1], hn[4 * i + 2], hn[4 * i + 3]);
         }
         const __nv_bfloat16* gb = reinterpret_cast<const __nv_bfloat16*>(gv);
@@ -243,7 +244,10 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
       const float* xv = S.xch + jl * kTileN;
       float o[16];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) o[i] = xv[c16 + i];
+      for (int i4 = 0; i4 < 4; ++i4) {
+        const float4 x4 = reinterpret_cast<const float4*>(xv + c16)[i4];
+        o[4 * i4] = x4.x; o[4 * i4 + 1] = x4.y; o[4 * i4 + 2] = x4.z; o[4 * i4 + 3] = x4.w;
+      }
       if (seg < 2) {
         // rotate-half RoPE: the 16 columns lie in one half of one head, and the
         // partner half of that head is in the same 128-row tile
@@ -255,11 +259,17 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
         for (int i = 0; i < 8; ++i)
           cs4[i] = make_float4(__uint_as_float(pre.w[i].x), __uint_as_float(pre.w[i].y), __uint_as_float(pre.w[i].z),
                                __uint_as_float(pre.w[i].w));
+        float pr[16];  // the partner half (pc: a multiple of 16 columns)
+#pragma unroll
+        for (int i4 = 0; i4 < 4; ++i4) {
+          const float4 x4 = reinterpret_cast<const float4*>(xv + pc)[i4];
+          pr[4 * i4] = x4.x; pr[4 * i4 + 1] = x4.y; pr[4 * i4 + 2] = x4.z; pr[4 * i4 + 3] = x4.w;
+        }
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const float c = (i & 1) ? cs4[i >> 1].z : cs4[i >> 1].x;
           const float sn = (i & 1) ? cs4[i >> 1].w : cs4[i >> 1].y;
-          const float p = xv[pc + i];
+          const float p = pr[i];
           o[i] = lo_half ? o[i] * c - p * sn : p * sn + o[i] * c;
         }
       }
@@ -298,8 +308,10 @@ static __device__ void epi_chunk(const GemmArgs& a, float (&v)[kEpiTok], int w_t
       if (m < M && n0 < a.seg_rows[0]) {
         const float* gp = S.xch + jl * kTileN + c8;
         float out[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) out[e] = silu(gp[e]) * gp[64 + e];
+        const float4 g0 = reinterpret_cast<const float4*>(gp)[0], g1 = reinterpret_cast<const float4*>(gp)[1];
+        const float4 u0 = reinterpret_cast<const float4*>(gp + 64)[0], u1 = reinterpret_cast<const float4*>(gp + 64)[1];
+        out[0] = silu(g0.x) * u0.x; out[1] = silu(g0.y) * u0.y; out[2] = silu(g0.z) * u0.z; out[3] = silu(g0.w) * u0.w;
+        out[4] = silu(g1.x) * u1.x; out[5] = silu(g1.y) * u1.y; out[6] = silu(g1.z) * u1.z; out[7] = silu(g1.w) * u1.w;
         if (n0 + 8 <= a.seg_rows[0]) {
           store_pair8(a.x_next, m, n0, a.x_rows, out);
         } else {

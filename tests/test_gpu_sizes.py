@@ -58,7 +58,7 @@ def test_batch16_ragged_c3_prompts_two_layers():
     """The batch-16 configuration at its own sizes (16 prompts of 128..2048
     tokens drawn from its seed, K = 6), two layers per model at full width:
     112 verify and up to 192 draft rows over contexts that differ by 16x.
-    The key splits are sized by the contexts' total (five splits here, more
+    The key splits are sized by the contexts' total (nine splits here, more
     units than two per SM), so the attention takes its two-buffer K/V ring
     with four CTAs per SM, and the long sequences' warp pairs split every
     chunk's keys; the clusters combine by the pull.  Three greedy steps."""
@@ -73,7 +73,7 @@ def test_batch16_ragged_c3_prompts_two_layers():
     bits = P.eng.attention_paths()
     print("paths", hex(bits), "cluster sizes", split_sizes(bits), "stats", P.stats)
     assert bits & PULL and bits & RING2
-    assert split_sizes(bits) == [5]
+    assert split_sizes(bits) == [9]
     assert P.eng.last_status() == 0
 
 
