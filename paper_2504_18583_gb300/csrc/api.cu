@@ -337,6 +337,7 @@ void run_gemm(pard_ctx* c, GemmArgs& a, int tt, cudaStream_t s) {
 // context).
 struct AttnGeom {
   int row_blocks, groups, n_split;
+  int nbuf;  // K/V chunk buffers of the attention kernel's form (4, or 2 for passes with many units)
 };
 AttnGeom attn_geometry(pard_ctx* c, int mi, int rows_per_seq, int batch) {
   const pard_model_cfg& cf = c->m[mi].cfg;
@@ -346,21 +347,31 @@ AttnGeom attn_geometry(pard_ctx* c, int mi, int rows_per_seq, int batch) {
   g.groups = batch * cf.n_kv_heads * g.row_blocks;
   const int n_kt = (c->lim.max_ctx + 31) / 32;  // 32-key chunks at the longest context
   g.n_split = std::max(1, std::min({c->attn_split_cap, n_kt, (2 * c->sm + g.groups - 1) / g.groups}));
-  if (batch > 1 && (int)c->ctx_est.size() >= batch) {
-    // Ragged contexts: the kernel lasts as long as the longest sequence's
-    // units, which walk its chunks / n_split each.  Split until that share is
-    // no longer than the average CTA's share of all units' chunks at four
-    // CTAs per SM (the two-buffer form such passes take; more splits only
-    // add per-CTA start-up and combine work).
-    long total = 0, longest = 0;
+  g.nbuf = 4;
+  long total = 0, longest = 0;
+  if (batch > 1 && (int)c->ctx_est.size() >= batch)
     for (int b = 0; b < batch; ++b) {
       const long ch = (c->ctx_est[b] + 31) / 32;
       total += ch;
       longest = std::max(longest, ch);
     }
+  const bool ragged = 2 * longest * batch > 3 * total;  // the longest context above 1.5 times the mean
+  const bool crowded = (long)g.groups * g.n_split > 2L * c->sm && longest >= 3L * g.n_split;
+  if (total > 0 && (ragged || crowded)) {
+    // Ragged contexts, where the kernel lasts as long as the longest
+    // sequence's units (its chunks / n_split each), or more units than two
+    // CTAs per SM that walk three chunks or more: such passes take the
+    // two-buffer ring (four CTAs per SM; its warp pairs split the keys of
+    // units with three chunks or more) and split until the longest
+    // sequence's share is no longer than the average CTA's share of all
+    // units' chunks at four CTAs per SM (even contexts: 4 x 152 / groups);
+    // more splits only add per-CTA start-up and combine work.  Measured on
+    // 512-token contexts: batch 4 (two chunks a unit) is faster with the
+    // four-buffer form, batch 8 and 16 with this one.
     total *= (long)cf.n_kv_heads * g.row_blocks;
-    const long bal = total > 0 ? (longest * 4 * c->sm + total - 1) / total : 1;
+    const long bal = (longest * 4 * c->sm + total - 1) / total;
     g.n_split = std::max<long>(g.n_split, std::min<long>({bal, (long)c->attn_split_cap, (long)n_kt}));
+    g.nbuf = 2;
   }
   return g;
 }
@@ -413,7 +424,7 @@ LayerPlan layer_plan(pard_ctx* c, int mi, int l, int rows_cap, int tt, int tt_gu
     a.batch = batch; a.hq = cf.n_q_heads; a.hkv = cf.n_kv_heads; a.hd = cf.head_dim;
     a.page_size = c->lim.page_size; a.n_pages = c->lim.n_pages;
     a.row_blocks = geo.row_blocks; a.n_split = geo.n_split;
-    a.nbuf = (long)geo.groups * geo.n_split > 2L * c->sm ? 2 : 4;
+    a.nbuf = geo.nbuf;
     a.scale = (float)(1.0 / std::sqrt((double)cf.head_dim));
     a.x_out = c->xo; a.x_rows = 2 * c->D.MC;
     a.status = c->status;
