@@ -287,9 +287,9 @@ int32_t pard_launch_count(pard_ctx* ctx);
  * the CTAs' key/value buffers: short contexts) or by a pull over distributed
  * shared memory (long contexts).  pard_attention_paths synchronises `stream`
  * and returns in *h_bits which forms ran since the last read (bit 0: push,
- * bit 1: pull, bit 2: the two-buffer K/V ring that passes with more units
- * than two per SM use, bit 3 + n: a cluster of n CTAs), then clears the
- * record.
+ * bit 1: pull, bit 2: the two-buffer K/V ring that passes with ragged
+ * contexts or with more multi-chunk units than two per SM take, bit 3 + n: a
+ * cluster of n CTAs), then clears the record.
  * pard_set_attention_split_cap limits the key splits of one unit to cap
  * CTAs (1..16; 0 restores the default 16) from the next pass on: the
  * launcher falls back to 8-CTA clusters on a GPU that cannot place 16, and a

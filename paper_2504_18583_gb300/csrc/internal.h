@@ -101,7 +101,7 @@ struct AttnArgs {
   int hq, hkv, hd, page_size, n_pages;
   int row_blocks;             // row blocks per sequence (grid.y / ...)
   int n_split;                // key splits
-  int nbuf;                   // K/V chunk buffers a CTA keeps (4, or 2 when many units share the SMs)
+  int nbuf;                   // K/V chunk buffers a CTA keeps (4, or 2 for ragged or crowded passes)
   float scale;
   __nv_bfloat16* x_out;       // packed [2*rows][hq*hd] hi/lo
   int x_rows;
